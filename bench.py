@@ -1,0 +1,508 @@
+#!/usr/bin/env python
+"""Benchmark of the draft-attention hot path (one drafting step per "step").
+
+A step drafts every level of one workload's draft chain/tree: per level, the
+new nodes' q/k/v are RoPE'd and appended, then they attend over
+[target prefix | draft KV] (kvshot_draft_append + kvshot_draft_attn, three
+kernels).  The default workload is the long-context multi-layer one (4
+sequences x 4 reused target layers = 16 caches of 32768 tokens, paged P=64,
+32-node depth-8 tree), the largest configuration; --workload selects another.
+
+Printed (rank 0, one JSON line): draft tokens/s (a token attending several
+reused layers counts once) over the timed steps with inputs resident in HBM,
+the achieved HBM bandwidth of the draft-attention call measured live with
+CUDA events (algorithmic bytes / time), the end-to-end rate through the C ABI
+with host buffers, the CPU oracle's rate on a bounded sample, GPU clocks.
+
+Multi-GPU: one process per GPU under torchrun runs an independent replica
+(the path has no exchange step); value = all ranks' tokens / max time.
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import hashlib
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2604_26412_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "draft-attn tokens/s and achieved HBM GB/s (fraction of GB300 peak) at 1 GPU"
+UNIT = "tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", type=int, default=5, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--mode", choices=["per_depth", "whole"], default="per_depth")
+    ap.add_argument("--kernel", choices=["auto", "cc", "mma"], default="auto")
+    ap.add_argument("--num-ctas", type=int, default=0)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-seconds", type=float, default=12.0)
+    ap.add_argument("--no-graph", action="store_true")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------- helpers
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return json.load(f), "measured"
+    except (OSError, ValueError):
+        return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2604_26412_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload, mode, kernel_hash):
+    """DRAM bytes per draft-attention call from a committed ncu summary, if it is
+    for the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    key = f"w{workload}-{mode}"
+    e = rec.get(key)
+    if not e or e.get("kernel_hash") != kernel_hash:
+        return None
+    return e.get("dram_bytes_per_call")
+
+
+def algorithmic_bytes(spec: wl.Spec, n_nodes: int, n_query: int, paged: bool) -> int:
+    """Bytes one draft-attention call must move: K and V of every visible-key
+    candidate (prefix + draft slots) once per KV head, q in, out and lse out,
+    the page-table entries and lengths read."""
+    D = spec.head_dim
+    kv = sum(spec.hkv * (L + n_nodes) * D * 2 * 2 for L in spec.seq_lens)
+    qo = 2 * spec.num_caches * n_query * spec.hq * D * 2
+    lse = spec.num_caches * n_query * spec.hq * 4
+    pt = sum(math.ceil(L / spec.page_size) * 4 for L in spec.seq_lens) if paged else 0
+    meta = spec.num_caches * 4 + (spec.num_seqs * n_nodes * 4 if spec.tree else 0)
+    return kv + qo + lse + pt + meta
+
+
+def algorithmic_flops(spec: wl.Spec, n_nodes: int, n_query: int) -> int:
+    return sum(4 * spec.hq * n_query * (L + n_nodes) * spec.head_dim for L in spec.seq_lens)
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled during the timed region."""
+
+    FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", "--query-gpu=" + ",".join(self.FIELDS), "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = [r for r in csv.reader(io.StringIO(out)) if len(r) == len(self.FIELDS)]
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.strip().lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------- CPU oracle
+
+def cpu_sample_spec(spec: wl.Spec) -> wl.Spec:
+    """One sequence of the workload (all its reused layers), same per-cache shapes."""
+    per = spec.layers
+    return wl.Spec(spec.name + "-seq0", 1, spec.layers, list(spec.seq_lens[:per]), list(spec.levels), spec.tree,
+                   spec.paged, page_size=spec.page_size, hq=spec.hq, hkv=spec.hkv, head_dim=spec.head_dim,
+                   max_fanout=spec.max_fanout, seed=spec.seed, rope_base=spec.rope_base)
+
+
+class OracleSample:
+    """The CPU oracle (as it stands) on one sequence of the workload: append +
+    attention of one drafting level per call."""
+
+    def __init__(self, spec: wl.Spec, mode: str, seed: int):
+        from oracle import oracle
+        self.oracle = oracle
+        oracle.build()
+        self.spec = cpu_sample_spec(spec)
+        self.inp = wl.make_inputs(self.spec, "cpu", seed=seed)
+        s, inp = self.spec, self.inp
+        self.tk, self.tv = wl.bf16_bits(inp.target_k), wl.bf16_bits(inp.target_v)
+        self.pt = inp.page_table.numpy() if inp.page_table is not None else None
+        self.lens = inp.seq_lens.numpy()
+        self.par = inp.tree_parent.numpy()
+        if mode == "per_depth":
+            self.levels = list(s.levels)
+            self.q = [wl.bf16_bits(x) for x in inp.q_in]
+            self.k = [wl.bf16_bits(x) for x in inp.k_in]
+            self.v = [wl.bf16_bits(x) for x in inp.v_in]
+            self.pos = [x.numpy() for x in inp.positions]
+        else:
+            self.levels = [s.n_nodes]
+            self.q = [wl.bf16_bits(torch.cat(inp.q_in, 1))]
+            self.k = [wl.bf16_bits(torch.cat(inp.k_in, 1))]
+            self.v = [wl.bf16_bits(torch.cat(inp.v_in, 1))]
+            self.pos = [torch.cat(inp.positions, 1).numpy()]
+        self.n0 = np.cumsum([0] + self.levels[:-1]).tolist()
+        C, D = s.num_caches, s.head_dim
+        self.dk = np.zeros((C, s.hkv, inp.n_max, D), np.uint16)
+        self.dv = self.dk.copy()
+        self.cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+        # fill the draft buffers once so any level can run alone
+        for i in range(len(self.levels)):
+            self._append(i)
+
+    def _append(self, i):
+        s, o = self.spec, self.oracle
+        d = o.make_desc(num_caches=s.num_caches, num_seqs=1, hq=s.hq, hkv=s.hkv, head_dim=s.head_dim, n_nodes=0,
+                        n_query=0, n_max=self.inp.n_max, tree=s.tree, l_cap=1)
+        return o.append(d, self.q[i], self.k[i], self.v[i], self.pos[i], self.n0[i], self.levels[i], s.rope_base,
+                        self.dk, self.dv)
+
+    def level(self, i) -> int:
+        """Append + attention of level i; returns the draft tokens it produced."""
+        s, o, inp = self.spec, self.oracle, self.inp
+        q_rot = self._append(i)
+        n_nodes = self.n0[i] + self.levels[i]
+        if s.paged:
+            d = o.make_desc(num_caches=s.num_caches, num_seqs=1, hq=s.hq, hkv=s.hkv, head_dim=s.head_dim,
+                            n_nodes=n_nodes, n_query=self.levels[i], n_max=inp.n_max, tree=s.tree, paged=True,
+                            page_size=s.page_size, max_pages_per_seq=self.pt.shape[1], num_pages=inp.num_pages)
+        else:
+            d = o.make_desc(num_caches=s.num_caches, num_seqs=1, hq=s.hq, hkv=s.hkv, head_dim=s.head_dim,
+                            n_nodes=n_nodes, n_query=self.levels[i], n_max=inp.n_max, tree=s.tree, l_cap=inp.l_cap)
+        o.attn(d, q_rot, self.tk, self.tv, self.pt, self.lens, self.dk, self.dv,
+               np.ascontiguousarray(self.par[:, :n_nodes]), nthreads=self.cores)
+        return self.levels[i]
+
+    def timed(self, budget_s: float):
+        """Run levels round-robin for about budget_s seconds; (tokens/s, description)."""
+        t0 = time.perf_counter()
+        tokens, calls, i = 0, 0, len(self.levels) - 1
+        while True:
+            tokens += self.level(i)
+            calls += 1
+            i = (i + 1) % len(self.levels)
+            if time.perf_counter() - t0 >= budget_s:
+                break
+        dt = time.perf_counter() - t0
+        sample = (f"{calls} drafting-level calls (append + attention) on 1 of {self.spec.num_seqs} sequence(s) "
+                  f"x {self.spec.layers} reused layer(s), fp64 oracle, {dt:.1f} s")
+        return tokens / dt, sample, dt
+
+
+# ---------------------------------------------------------------- our arm
+
+def run_ours(args, world, rank, local):
+    from paper_2604_26412_gb300 import kvshot
+    from paper_2604_26412_gb300.step import DraftStep
+
+    dev = torch.device("cuda", torch.cuda.current_device())
+    spec = wl.config(args.workload, seed=args.seed)
+    inp = wl.make_inputs(spec, dev, seed=args.seed + 1000 * rank)
+    flags = {"auto": 0, "cc": kvshot.KVSHOT_FORCE_CC, "mma": kvshot.KVSHOT_FORCE_MMA}[args.kernel]
+    step = DraftStep(inp, mode=args.mode, flags=flags, num_ctas=args.num_ctas)
+    paged = inp.page_table is not None
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            step.run()
+    torch.cuda.synchronize()
+    if step.error_code() != 0:
+        raise RuntimeError(f"device error {step.error_code()}")
+
+    graph = None
+    if not args.no_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            step.run()
+        with torch.cuda.stream(stream):
+            for _ in range(2):
+                graph.replay()
+        torch.cuda.synchronize()
+
+    # ---- timed region: K steps, inputs resident in HBM (larger than L2 for the long-prefix workloads)
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t_start.record(stream)
+        for _ in range(args.steps):
+            if graph is not None:
+                graph.replay()
+            else:
+                step.run()
+        t_end.record(stream)
+    torch.cuda.synchronize()
+    clock_info = clocks.stop()
+    barrier(world)
+    ms_total = max_over_ranks(t_start.elapsed_time(t_end), world)
+    ms_per_step = ms_total / args.steps
+    tokens_per_step = step.tokens
+    value = tokens_per_step * world * args.steps / (ms_total / 1e3)
+
+    # ---- live roofline of the draft-attention call (attention + merge kernels), per level
+    levels = step.levels
+    n0s = np.cumsum([0] + levels[:-1]).tolist()
+    reps = max(3, min(50, int(2000 / max(ms_per_step, 1e-3) / len(levels))))
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in levels]
+          for _ in range(reps)]
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(2e7))  # keep the GPU busy while the host enqueues the calls
+        for r in range(reps):
+            for i in range(len(levels)):
+                ev[r][i][0].record(stream)
+                kvshot.draft_attn(step.descs[i], step.q_rot[i], inp.target_k, inp.target_v, inp.page_table,
+                                  inp.seq_lens, step.draft_k, step.draft_v, step.parents[i], step.out[i], step.lse[i],
+                                  stream)
+                ev[r][i][1].record(stream)
+    torch.cuda.synchronize()
+    call_ms = [statistics.mean(ev[r][i][0].elapsed_time(ev[r][i][1]) for r in range(reps)) for i in range(len(levels))]
+    call_bytes = [algorithmic_bytes(spec, n0s[i] + levels[i], levels[i], paged) for i in range(len(levels))]
+    call_flops = [algorithmic_flops(spec, n0s[i] + levels[i], levels[i]) for i in range(len(levels))]
+    achieved_gbs = sum(call_bytes) / (sum(call_ms) / 1e3) / 1e9
+    achieved_tflops = sum(call_flops) / (sum(call_ms) / 1e3) / 1e12
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    khash = kernel_source_hash()
+    traffic = recorded_traffic(args.workload, args.mode, khash)
+    rows_per_head = spec.hq // spec.hkv * max(levels)
+    roofline = {
+        "bound": "hbm",
+        "kernel": "kvshot_draft_attn (attention + merge kernels)",
+        "achieved": round(achieved_gbs, 1),
+        "peak": hbm_peak,
+        "unit": "GB/s",
+        "frac": round(achieved_gbs / hbm_peak, 4),
+        "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6.8 TB/s",
+        "traffic": traffic,
+        "algorithmic_bytes_per_call": int(statistics.mean(call_bytes)),
+        "call_us": round(statistics.mean(call_ms) * 1e3, 2),
+        "per_level_us": [round(x * 1e3, 2) for x in call_ms],
+        "achieved_tflops": round(achieved_tflops, 2),
+        "max_rows_per_kv_head": rows_per_head,
+        "kernel_hash": khash,
+    }
+
+    # ---- end to end through the C ABI with host buffers (pinned), copies in the timed region
+    e2e = run_e2e(args, step, inp, stream, world)
+
+    gpu_launches = 3 * len(levels) * args.steps
+    result = {
+        "metric": METRIC,
+        "value": round(value, 1),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) K/V, N(0,1)/sqrt(128) q; shapes of the paper's Qwen3-8B runs)",
+        "config": {
+            "workload": spec.name,
+            "mode": args.mode,
+            "num_seqs": spec.num_seqs,
+            "reused_layers": spec.layers,
+            "num_caches": spec.num_caches,
+            "prefix_lens": "ragged U[512,8192]" if args.workload == 4 else spec.seq_lens[0],
+            "draft_levels": list(spec.levels),
+            "tree": spec.tree,
+            "layout": f"paged P={spec.page_size}" if paged else "contiguous",
+            "gqa": f"{spec.hq}/{spec.hkv}",
+            "head_dim": spec.head_dim,
+            "tokens_per_step": tokens_per_step,
+            "cuda_graph": graph is not None,
+            "l2": "inputs larger than L2 (no flush)" if sum(call_bytes) / len(call_bytes) > 2 * 129e6
+                  else "inputs smaller than L2 (not flushed: latency-bound workload)",
+            "parallelism": f"replicas x{world}",
+        },
+        "roofline": roofline,
+        "e2e": e2e,
+        "clocks": clock_info,
+        "gpu_launches": gpu_launches,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        samp = OracleSample(spec, args.mode, args.seed)
+        v, desc, _ = samp.timed(args.cpu_sample_seconds)
+        result["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": samp.cores, "kind": "oracle",
+                                  "sample": desc}
+    return result
+
+
+def run_e2e(args, step, inp, stream, world):
+    """Same steps through the C ABI, with the per-step inputs copied from pinned
+    host buffers and the outputs copied back inside the timed region."""
+    host_in = []
+    dev_in = []
+    for lst in (step.q_in, step.k_in, step.v_in, step.pos):
+        for t in lst:
+            host_in.append(t.cpu().pin_memory())
+            dev_in.append(t)
+    for t in step.parents + [inp.seq_lens] + ([inp.page_table] if inp.page_table is not None else []):
+        host_in.append(t.cpu().pin_memory())
+        dev_in.append(t)
+    host_out = [t.cpu().pin_memory() for t in step.out + step.lse]
+    dev_out = step.out + step.lse
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
+    steps = max(3, min(args.steps, 100))
+    torch.cuda.synchronize()
+    barrier(world)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        a.record(stream)
+        for _ in range(steps):
+            for h, d in zip(host_in, dev_in):
+                d.copy_(h, non_blocking=True)
+            step.run()
+            for d, h in zip(dev_out, host_out):
+                h.copy_(d, non_blocking=True)
+        b.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(a.elapsed_time(b), world)
+    value = step.tokens * world * steps / (ms / 1e3)
+    return {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "steps": steps, "api": "kvshot_draft_append + kvshot_draft_attn via ctypes, no CUDA graph"}
+
+
+# --------------------------------------------------------- reference arm
+
+def run_reference(args):
+    """The CPU fp64 oracle as it stands, timed on the host cores; each step is
+    one drafting level (append + attention) of one sequence of the workload."""
+    spec = wl.config(args.workload, seed=args.seed)
+    samp = OracleSample(spec, args.mode, args.seed)
+    for w in range(args.warmup):
+        samp.level(w % len(samp.levels))
+    t0 = time.perf_counter()
+    tokens = 0
+    for k in range(args.steps):
+        tokens += samp.level(k % len(samp.levels))
+    dt = time.perf_counter() - t0
+    value = tokens / dt
+    sample = (f"{args.steps} drafting-level calls (append + attention) on 1 of {spec.num_seqs} sequence(s) x "
+              f"{spec.layers} reused layer(s), fp64 oracle")
+    return {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": round(value, 3),
+        "unit": UNIT,
+        "n_gpus": args.gpus,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(dt / args.steps * 1e3, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic (seeded; same shapes as the GPU arm)",
+        "config": {"workload": spec.name, "mode": args.mode, "parallelism": "host cores"},
+        "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": samp.cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        rank = int(os.environ.get("RANK", "0"))
+        if rank != 0:
+            return
+        print(json.dumps(run_reference(args)), flush=True)
+        return
+    world, rank, local = dist_setup()
+    result = run_ours(args, world, rank, local)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,168 @@
+/*
+ * kvshot.h -- C ABI of libkvshot, GB300 (sm_103a) draft attention for
+ * KV-reuse speculative drafting.
+ *
+ * The drafter of a KV-reuse speculative decoder re-attends, with its own
+ * query, to the target model's key/value cache instead of (or next to) the
+ * target's hidden state: a' = sum_i alpha_i(q') v_i with
+ * alpha_i(q') = softmax_i(q'^T k_i)  (arXiv 2604.26412, Sec. 2.2,
+ * Eq. "kv-reattention").  Its memory M_i holds the target K/V of the verified
+ * prefix (j <= t) followed by K/V the drafter produced for its own earlier
+ * draft positions (j > t)  (Sec. 3.4, Eq. "cross-attn"; App. B,
+ * "Cross-attention memory").  The same attention step serves the KV-only
+ * drafter (Sec. 3.2) and the cross-attention branch o_i of the hybrid
+ * gated-delta drafter (Sec. 3.4).  Draft positions form a chain (K draft
+ * tokens drafted one after another, Sec. 4.2) or a tree (tree verification
+ * with a (8, 10, 60) draft tree, Sec. 3.1 and 3.5); a draft node sees every
+ * verified prefix token plus itself and its ancestors among the draft nodes.
+ *
+ * Conventions for every entry point:
+ *  - All tensor pointers are DEVICE pointers owned by the caller.  The
+ *    library never allocates; scratch space is the caller's workspace.
+ *  - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream).  Nothing synchronises the host.
+ *  - Argument errors are found on the host, before anything is enqueued, and
+ *    returned as a kvshot_status; nothing is launched then.
+ *  - Errors only visible on the device (a page id outside the pool, a
+ *    sequence length above the stated bound, a parent index that is not an
+ *    earlier node, a pipeline wait that timed out) are recorded in
+ *    desc->err_flag (if non-NULL): the first error code is stored with an
+ *    atomic compare-and-swap from 0.  Outputs of the affected call are then
+ *    unspecified.  No kernel traps.
+ *  - bf16 tensors are row-major with the innermost dimension head_dim (= 128).
+ */
+#ifndef KVSHOT_H
+#define KVSHOT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* kvshot_stream_t; /* same handle type as cudaStream_t */
+
+typedef enum kvshot_status {
+  KVSHOT_OK = 0,
+  KVSHOT_ERR_NULL = 1,          /* a required pointer is NULL */
+  KVSHOT_ERR_SHAPE = 2,         /* inconsistent or out-of-range sizes in the descriptor */
+  KVSHOT_ERR_ALIGN = 3,         /* a pointer is not aligned as stated below */
+  KVSHOT_ERR_UNSUPPORTED = 4,   /* valid but outside this build (head_dim != 128, tree with > 64 nodes, ...) */
+  KVSHOT_ERR_TREE = 5,          /* (device) tree_parent[i] is not in [-1, i) */
+  KVSHOT_ERR_WORKSPACE = 6,     /* workspace missing, misaligned or smaller than the size query returns */
+  KVSHOT_ERR_CUDA = 7,          /* a CUDA runtime/driver call failed (tensor map encode, launch) */
+  KVSHOT_ERR_DEVICE_BOUNDS = 8, /* (device) page id outside the pool or seq_len above its bound */
+  KVSHOT_ERR_TIMEOUT = 9        /* (device) a pipeline wait gave up after its time limit */
+} kvshot_status;
+
+/* desc->flags */
+#define KVSHOT_TREE 0x1u       /* draft nodes form a tree given by tree_parent (else a chain) */
+#define KVSHOT_FORCE_CC 0x2u   /* use the CUDA-core kernel whatever the row count (measurement aid) */
+#define KVSHOT_FORCE_MMA 0x4u  /* use the tensor-core kernel whatever the row count (measurement aid) */
+
+/*
+ * Problem descriptor shared by kvshot_draft_attn and kvshot_draft_append.
+ *
+ * A "cache" is one independent KV cache: one sequence when one target layer
+ * is reused, or one (sequence, reused target layer) pair when several target
+ * layers are attended separately (KV-only head concatenation, Sec. 3.2).
+ * Caches of one sequence are consecutive and share that sequence's draft tree.
+ */
+typedef struct kvshot_attn_desc {
+  int32_t num_caches;        /* C >= 1 (<= 1024) */
+  int32_t num_seqs;          /* B >= 1, C % B == 0; cache c belongs to sequence c / (C / B) */
+  int32_t hq;                /* query heads */
+  int32_t hkv;               /* KV heads; hq % hkv == 0 (GQA group G = hq / hkv) */
+  int32_t head_dim;          /* must be 128 */
+  int32_t page_size;         /* paged layout: tokens per page: 8, 16, 32, 64, 128, 192 or 256 */
+  int32_t max_pages_per_seq; /* paged layout: row stride of page_table */
+  int32_t num_pages;         /* paged layout: pages in the target_k / target_v pools */
+  int32_t l_cap;             /* contiguous layout: token capacity per (cache, KV head) */
+  int32_t max_seq_len;       /* host-known upper bound on every seq_lens[c]; sizes the work plan */
+  int32_t n_nodes;           /* N: draft nodes present; draft slots 0..N-1 hold their K/V */
+  int32_t n_query;           /* Nq: the last Nq draft nodes are the query rows (Nq <= N) */
+  int32_t n_max;             /* draft buffer capacity in slots (N <= n_max) */
+  float scale;               /* softmax scale on q.k; 0 selects 1/sqrt(head_dim) */
+  uint32_t flags;            /* KVSHOT_TREE, KVSHOT_FORCE_CC, KVSHOT_FORCE_MMA */
+  int32_t num_ctas;          /* persistent CTAs to launch; 0 = one full wave on this GPU */
+  void* workspace;           /* device scratch, 256-byte aligned; see kvshot_draft_attn_workspace_size */
+  size_t workspace_bytes;
+  int32_t* err_flag;         /* optional device int32, 0 before the call; see conventions above */
+} kvshot_attn_desc;
+
+/*
+ * Bytes of workspace kvshot_draft_attn needs for `desc` on the current device
+ * (partial softmax states of work pieces that straddle CTAs, plus the work
+ * plan).  Returns 0 if the descriptor is invalid.  The size depends on the
+ * shape fields, flags, num_ctas and the device's SM count, not on pointers.
+ */
+size_t kvshot_draft_attn_workspace_size(const kvshot_attn_desc* desc);
+
+/*
+ * Draft attention.  For every cache c, query row n_local in [0, Nq) (draft
+ * node n = N - Nq + n_local) and query head h (KV head h / G):
+ *
+ *   keys  = { prefix tokens j in [0, L_c) }  U  { draft slots m : m == n or m is an ancestor of n }
+ *   s_k   = scale * q . k_k
+ *   lse   = log sum_k exp(s_k)                          (natural log)
+ *   out   = sum_k exp(s_k - lse) v_k                    (fp32 accumulate, rounded to bf16)
+ *
+ * where L_c = seq_lens[c] (Sec. 2.2 Eq. "kv-reattention" over M_i of Sec. 3.4 / App. B).
+ * A chain (flags without KVSHOT_TREE) means node n's ancestors are 0..n-1.
+ *
+ * q:           [C, Nq, hq, 128] bf16, 16-byte aligned.
+ * target_k/v:  paged (page_table != NULL): [num_pages, hkv, page_size, 128] bf16;
+ *              contiguous (page_table == NULL): [C, hkv, l_cap, 128] bf16.  16-byte aligned.
+ *              Rows past L_c may hold anything (NaN included); they are never used.
+ * page_table:  [C, max_pages_per_seq] int32; entry p of cache c is the pool page of tokens
+ *              [p * page_size, (p + 1) * page_size).  Only the first ceil(L_c / page_size) entries are read.
+ * seq_lens:    [C] int32, 0 <= L_c <= min(max_seq_len, capacity).
+ * draft_k/v:   [C, hkv, n_max, 128] bf16, 16-byte aligned; slots 0..N-1 are read.
+ * tree_parent: [B, N] int32, parent[i] in [-1, i) (-1 = child of the last verified token);
+ *              read only with KVSHOT_TREE (then N <= 64).  May be NULL for a chain.
+ * out:         [C, Nq, hq, 128] bf16, 16-byte aligned, must not alias any input.
+ * lse:         [C, Nq, hq] fp32 (natural log), 4-byte aligned.
+ * Nq == 0 is a no-op returning KVSHOT_OK.
+ */
+kvshot_status kvshot_draft_attn(const kvshot_attn_desc* desc, const void* q, const void* target_k,
+                                const void* target_v, const int32_t* page_table, const int32_t* seq_lens,
+                                const void* draft_k, const void* draft_v, const int32_t* tree_parent,
+                                void* out, float* lse, kvshot_stream_t stream);
+
+/*
+ * Draft append with RoPE: the drafter's new K/V for draft positions j > t
+ * enter M_i (App. B: "the drafter generates its own KV via learned
+ * projections"; the projections themselves are upstream GEMMs), with rotary
+ * position embedding applied to q and k (RoPE re-application, Sec. 3.2).
+ *
+ * For cache c and new node i in [0, n_new) at position pos = positions[c, i]:
+ *   theta_j = pos * rope_base^(-2j / 128),  j in [0, 64)
+ *   rot(x)[j]      = x[j] cos(theta_j) - x[j + 64] sin(theta_j)
+ *   rot(x)[j + 64] = x[j + 64] cos(theta_j) + x[j] sin(theta_j)
+ *   q_out[c, i, h]              = bf16(rot(q_in[c, i, h]))      for h < hq
+ *   draft_k[c, kh, n0 + i]      = bf16(rot(k_in[c, i, kh]))     for kh < hkv
+ *   draft_v[c, kh, n0 + i]      = v_in[c, i, kh]                (copied bit for bit)
+ * Angles and rotations are computed in fp64 and rounded once to bf16 (nearest even).
+ *
+ * q_in:  [C, n_new, hq, 128] bf16; k_in, v_in: [C, n_new, hkv, 128] bf16; positions: [C, n_new] int32 >= 0.
+ * draft_k/v: [C, hkv, n_max, 128] bf16 (desc->n_max); requires 0 <= n0 and n0 + n_new <= n_max.
+ * q_out: [C, n_new, hq, 128] bf16; may equal q_in (in place) but must not partially overlap it.
+ * All bf16 pointers 16-byte aligned.  Only num_caches, hq, hkv, head_dim and n_max of desc are read.
+ * n_new == 0 is a no-op returning KVSHOT_OK.
+ */
+kvshot_status kvshot_draft_append(const kvshot_attn_desc* desc, const void* q_in, const void* k_in,
+                                  const void* v_in, const int32_t* positions, int32_t n0, int32_t n_new,
+                                  float rope_base, void* draft_k, void* draft_v, void* q_out,
+                                  kvshot_stream_t stream);
+
+/* Static description of a status code (never NULL). */
+const char* kvshot_status_string(kvshot_status status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int32_t kvshot_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVSHOT_H */

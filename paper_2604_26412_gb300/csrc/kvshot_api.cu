@@ -1,0 +1,297 @@
+// kvshot_api.cu -- host side of libkvshot's C ABI: argument validation, the
+// work planner (kernel choice, row blocks, persistent grid, workspace
+// layout), TMA tensor-map encoding and the launches.  No host synchronisation,
+// no allocation.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <climits>
+#include <cmath>
+#include <mutex>
+
+#include "kvshot_internal.h"
+
+namespace kvshot {
+
+// Defined in the kernel translation units.
+cudaError_t attn_cc_occupancy(int C, int* ctas_per_sm);
+cudaError_t attn_mma_occupancy(int m_tiles, int C, int* ctas_per_sm);
+
+namespace {
+
+constexpr int kVersion = 100;  // 0.1.0
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// 2-D view [rows, 128] of a bf16 tensor, boxes of {64 dims, box_rows rows},
+// 128-byte swizzle (matches tile_off in kvshot_attn_common.cuh).
+bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(kHeadDim) * 2};
+  const cuuint32_t box[2] = {64, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct Plan {
+  bool mma;
+  int m_tiles;        // mma path
+  int rows_per_unit;
+  int row_blocks;
+  int units;
+  int num_ctas;
+  int len_bound;
+  int draft_tiles;
+  size_t off_lse, off_o, bytes;
+};
+
+int sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  if (dev >= 0 && dev < 64) cached[dev] = n;
+  return n;
+}
+
+// Checks that do not depend on the cache layout.
+kvshot_status check_common(const kvshot_attn_desc* d) {
+  if (d == nullptr) return KVSHOT_ERR_NULL;
+  if (d->num_caches < 1 || d->num_seqs < 1 || d->num_caches % d->num_seqs != 0) return KVSHOT_ERR_SHAPE;
+  if (d->num_caches > kMaxCaches) return KVSHOT_ERR_UNSUPPORTED;
+  if (d->hq < 1 || d->hkv < 1 || d->hq % d->hkv != 0) return KVSHOT_ERR_SHAPE;
+  if (d->head_dim != kHeadDim) return KVSHOT_ERR_UNSUPPORTED;
+  if (d->n_nodes < 0 || d->n_query < 0 || d->n_query > d->n_nodes || d->n_nodes > d->n_max) return KVSHOT_ERR_SHAPE;
+  if (d->max_seq_len < 0) return KVSHOT_ERR_SHAPE;
+  if (!std::isfinite(d->scale)) return KVSHOT_ERR_SHAPE;
+  const uint32_t known = KVSHOT_TREE | KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA;
+  if ((d->flags & ~known) != 0) return KVSHOT_ERR_SHAPE;
+  if ((d->flags & KVSHOT_FORCE_CC) && (d->flags & KVSHOT_FORCE_MMA)) return KVSHOT_ERR_SHAPE;
+  if ((d->flags & KVSHOT_TREE) && d->n_nodes > kMaxTreeNodes) return KVSHOT_ERR_UNSUPPORTED;
+  if (d->num_ctas < 0) return KVSHOT_ERR_SHAPE;
+  if (static_cast<int64_t>(d->num_caches) * d->hkv * d->n_max >= INT_MAX) return KVSHOT_ERR_UNSUPPORTED;
+  return KVSHOT_OK;
+}
+
+kvshot_status check_attn_desc(const kvshot_attn_desc* d, bool paged) {
+  if (kvshot_status st = check_common(d)) return st;
+  if (paged) {
+    // A 64-key tile must cover whole pages or lie inside one page: P in {8, 16, 32, 64, 128, 192, 256}.
+    const int P = d->page_size;
+    if (P < 8 || P > 256 || !(kTileKeys % P == 0 || P % kTileKeys == 0)) return KVSHOT_ERR_UNSUPPORTED;
+    if (d->max_pages_per_seq < 1 || d->num_pages < 1) return KVSHOT_ERR_SHAPE;
+    const int64_t rows = static_cast<int64_t>(d->num_pages) * d->hkv * d->page_size;
+    if (rows >= INT_MAX) return KVSHOT_ERR_UNSUPPORTED;
+    if (static_cast<int64_t>(d->num_caches) * d->max_pages_per_seq >= INT_MAX) return KVSHOT_ERR_UNSUPPORTED;
+  } else {
+    if (d->l_cap < 1) return KVSHOT_ERR_SHAPE;
+    if (static_cast<int64_t>(d->num_caches) * d->hkv * d->l_cap >= INT_MAX) return KVSHOT_ERR_UNSUPPORTED;
+  }
+  return KVSHOT_OK;
+}
+
+kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
+  const int G = d->hq / d->hkv;
+  const int rows = G * d->n_query;
+  const bool force_cc = d->flags & KVSHOT_FORCE_CC, force_mma = d->flags & KVSHOT_FORCE_MMA;
+  pl->mma = force_mma || (!force_cc && rows > kCcRows);
+  if (pl->mma) {
+    pl->m_tiles = std::min(kMmaMaxTiles, std::max(1, (rows + 15) / 16));
+    pl->rows_per_unit = 16 * pl->m_tiles;
+  } else {
+    pl->m_tiles = 0;
+    pl->rows_per_unit = kCcRows;
+  }
+  pl->row_blocks = std::max(1, (rows + pl->rows_per_unit - 1) / pl->rows_per_unit);
+  const int64_t units = static_cast<int64_t>(d->num_caches) * d->hkv * pl->row_blocks;
+  const int64_t cap = paged ? static_cast<int64_t>(d->max_pages_per_seq) * d->page_size : d->l_cap;
+  pl->len_bound = static_cast<int>(std::min<int64_t>(d->max_seq_len, cap));
+  pl->draft_tiles = (d->n_nodes + kTileKeys - 1) / kTileKeys;
+  // Upper bound on the tiles of any call with this descriptor (independent of the layout, so the
+  // workspace size query and the call agree).
+  const int64_t max_tiles =
+      units * ((static_cast<int64_t>(d->max_seq_len) + kTileKeys - 1) / kTileKeys + pl->draft_tiles);
+  if (units >= INT_MAX / 2 || max_tiles >= INT_MAX / 2) return KVSHOT_ERR_UNSUPPORTED;
+  pl->units = static_cast<int>(units);
+  int grid = d->num_ctas;
+  if (grid == 0) {
+    int per_sm = 0;
+    const cudaError_t e = pl->mma ? attn_mma_occupancy(pl->m_tiles, d->num_caches, &per_sm)
+                                  : attn_cc_occupancy(d->num_caches, &per_sm);
+    const int sms = sm_count();
+    if (e != cudaSuccess || per_sm < 1 || sms < 1) return KVSHOT_ERR_CUDA;
+    grid = sms * per_sm;
+  }
+  grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(grid, std::max<int64_t>(1, max_tiles))));
+  pl->num_ctas = grid;
+  const size_t slots = static_cast<size_t>(pl->units) + grid;
+  pl->off_lse = round_up(sizeof(int32_t) * (d->num_caches + 1), 256);
+  pl->off_o = pl->off_lse + round_up(sizeof(float) * slots * pl->rows_per_unit, 256);
+  pl->bytes = pl->off_o + sizeof(float) * slots * pl->rows_per_unit * kHeadDim;
+  return KVSHOT_OK;
+}
+
+}  // namespace
+}  // namespace kvshot
+
+using namespace kvshot;
+
+extern "C" const char* kvshot_status_string(kvshot_status s) {
+  switch (s) {
+    case KVSHOT_OK: return "ok";
+    case KVSHOT_ERR_NULL: return "a required pointer is NULL";
+    case KVSHOT_ERR_SHAPE: return "inconsistent or out-of-range sizes";
+    case KVSHOT_ERR_ALIGN: return "misaligned pointer";
+    case KVSHOT_ERR_UNSUPPORTED: return "valid but unsupported by this build";
+    case KVSHOT_ERR_TREE: return "tree_parent entry is not an earlier node or -1";
+    case KVSHOT_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case KVSHOT_ERR_CUDA: return "CUDA call failed";
+    case KVSHOT_ERR_DEVICE_BOUNDS: return "page id or sequence length out of bounds";
+    case KVSHOT_ERR_TIMEOUT: return "device pipeline wait timed out";
+  }
+  return "unknown status";
+}
+
+extern "C" int32_t kvshot_version(void) { return kVersion; }
+
+extern "C" size_t kvshot_draft_attn_workspace_size(const kvshot_attn_desc* d) {
+  if (d == nullptr || check_common(d) != KVSHOT_OK) return 0;
+  if (d->n_query == 0) return 256;
+  Plan pl;
+  if (make_plan(d, false, &pl) != KVSHOT_OK) return 0;  // the size does not depend on the layout
+  return pl.bytes;
+}
+
+extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void* q, const void* target_k,
+                                           const void* target_v, const int32_t* page_table,
+                                           const int32_t* seq_lens, const void* draft_k, const void* draft_v,
+                                           const int32_t* tree_parent, void* out, float* lse,
+                                           kvshot_stream_t stream) {
+  const bool paged = page_table != nullptr;
+  if (kvshot_status st = check_attn_desc(d, paged)) return st;
+  if (d->n_query == 0) return KVSHOT_OK;
+  const bool tree = d->flags & KVSHOT_TREE;
+  if (!q || !target_k || !target_v || !seq_lens || !draft_k || !draft_v || !out || !lse) return KVSHOT_ERR_NULL;
+  if (tree && !tree_parent) return KVSHOT_ERR_NULL;
+  if (!aligned(q, 16) || !aligned(target_k, 16) || !aligned(target_v, 16) || !aligned(draft_k, 16) ||
+      !aligned(draft_v, 16) || !aligned(out, 16) || !aligned(lse, 4) || !aligned(seq_lens, 4) ||
+      (paged && !aligned(page_table, 4)) || (tree && !aligned(tree_parent, 4)))
+    return KVSHOT_ERR_ALIGN;
+  Plan pl;
+  if (kvshot_status st = make_plan(d, paged, &pl)) return st;
+  if (d->workspace == nullptr || !aligned(d->workspace, 256) || d->workspace_bytes < pl.bytes)
+    return KVSHOT_ERR_WORKSPACE;
+
+  TensorMaps maps;
+  const uint64_t trows = paged ? static_cast<uint64_t>(d->num_pages) * d->hkv * d->page_size
+                               : static_cast<uint64_t>(d->num_caches) * d->hkv * d->l_cap;
+  const uint32_t tbox = paged ? static_cast<uint32_t>(std::min(d->page_size, kTileKeys)) : kTileKeys;
+  const uint64_t drows = static_cast<uint64_t>(d->num_caches) * d->hkv * d->n_max;
+  if (!encode_rows(&maps.tk, target_k, trows, tbox) || !encode_rows(&maps.tv, target_v, trows, tbox) ||
+      !encode_rows(&maps.dk, draft_k, drows, kDraftBoxRows) || !encode_rows(&maps.dv, draft_v, drows, kDraftBoxRows))
+    return KVSHOT_ERR_CUDA;
+
+  AttnParams p;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.lse = lse;
+  p.page_table = page_table;
+  p.seq_lens = seq_lens;
+  p.tree_parent = tree_parent;
+  p.err = d->err_flag;
+  uint8_t* ws = static_cast<uint8_t*>(d->workspace);
+  p.ws_meta = reinterpret_cast<int32_t*>(ws);
+  p.ws_lse = reinterpret_cast<float*>(ws + pl.off_lse);
+  p.ws_o = reinterpret_cast<float*>(ws + pl.off_o);
+  p.C = d->num_caches;
+  p.B = d->num_seqs;
+  p.hq = d->hq;
+  p.hkv = d->hkv;
+  p.G = d->hq / d->hkv;
+  p.rows_total = p.G * d->n_query;
+  p.rows_per_unit = pl.rows_per_unit;
+  p.row_blocks = pl.row_blocks;
+  p.paged = paged ? 1 : 0;
+  p.page_size = paged ? d->page_size : kTileKeys;
+  p.max_pages = paged ? d->max_pages_per_seq : 0;
+  p.num_pages = paged ? d->num_pages : 0;
+  p.l_cap = paged ? 0 : d->l_cap;
+  p.box_rows = static_cast<int>(tbox);
+  p.len_bound = pl.len_bound;
+  p.N = d->n_nodes;
+  p.Nq = d->n_query;
+  p.n_max = d->n_max;
+  p.tree = tree ? 1 : 0;
+  p.draft_tiles = pl.draft_tiles;
+  const double scale = d->scale != 0.f ? static_cast<double>(d->scale) : 1.0 / std::sqrt(static_cast<double>(kHeadDim));
+  p.qscale = static_cast<float>(scale * 1.4426950408889634);
+  p.num_ctas = pl.num_ctas;
+
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = pl.mma ? launch_attn_mma(p, maps, pl.m_tiles, s) : launch_attn_cc(p, maps, s);
+  if (e != cudaSuccess) return KVSHOT_ERR_CUDA;
+  e = launch_merge(p, s);
+  return e == cudaSuccess ? KVSHOT_OK : KVSHOT_ERR_CUDA;
+}
+
+extern "C" kvshot_status kvshot_draft_append(const kvshot_attn_desc* d, const void* q_in, const void* k_in,
+                                             const void* v_in, const int32_t* positions, int32_t n0,
+                                             int32_t n_new, float rope_base, void* draft_k, void* draft_v,
+                                             void* q_out, kvshot_stream_t stream) {
+  if (d == nullptr) return KVSHOT_ERR_NULL;
+  if (d->num_caches < 1 || d->hq < 1 || d->hkv < 1 || d->n_max < 0) return KVSHOT_ERR_SHAPE;
+  if (d->head_dim != kHeadDim) return KVSHOT_ERR_UNSUPPORTED;
+  if (n0 < 0 || n_new < 0 || static_cast<int64_t>(n0) + n_new > d->n_max) return KVSHOT_ERR_SHAPE;
+  if (!(rope_base > 0.f) || !std::isfinite(rope_base)) return KVSHOT_ERR_SHAPE;
+  if (n_new == 0) return KVSHOT_OK;
+  if (static_cast<int64_t>(d->num_caches) * n_new >= INT_MAX ||
+      static_cast<int64_t>(d->num_caches) * d->hkv * d->n_max >= INT_MAX)
+    return KVSHOT_ERR_UNSUPPORTED;
+  if (!q_in || !k_in || !v_in || !positions || !draft_k || !draft_v || !q_out) return KVSHOT_ERR_NULL;
+  if (!aligned(q_in, 16) || !aligned(k_in, 16) || !aligned(v_in, 16) || !aligned(draft_k, 16) ||
+      !aligned(draft_v, 16) || !aligned(q_out, 16) || !aligned(positions, 4))
+    return KVSHOT_ERR_ALIGN;
+  // q_out may be q_in exactly, but must not partially overlap it.
+  const size_t qbytes = static_cast<size_t>(d->num_caches) * n_new * d->hq * kHeadDim * 2;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(q_in), b = reinterpret_cast<uintptr_t>(q_out);
+  if (a != b && a < b + qbytes && b < a + qbytes) return KVSHOT_ERR_SHAPE;
+  AppendParams ap;
+  ap.q_in = static_cast<const __nv_bfloat16*>(q_in);
+  ap.k_in = static_cast<const __nv_bfloat16*>(k_in);
+  ap.v_in = static_cast<const __nv_bfloat16*>(v_in);
+  ap.positions = positions;
+  ap.draft_k = static_cast<__nv_bfloat16*>(draft_k);
+  ap.draft_v = static_cast<__nv_bfloat16*>(draft_v);
+  ap.q_out = static_cast<__nv_bfloat16*>(q_out);
+  ap.C = d->num_caches;
+  ap.hq = d->hq;
+  ap.hkv = d->hkv;
+  ap.n_max = d->n_max;
+  ap.n0 = n0;
+  ap.n_new = n_new;
+  for (int j = 0; j < kHeadDim / 2; ++j)
+    ap.inv_freq[j] = std::pow(static_cast<double>(rope_base), -2.0 * j / kHeadDim);
+  const cudaError_t e = launch_append(ap, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? KVSHOT_OK : KVSHOT_ERR_CUDA;
+}

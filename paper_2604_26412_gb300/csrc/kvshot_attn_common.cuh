@@ -1,0 +1,443 @@
+// kvshot_attn_common.cuh -- device building blocks shared by the draft
+// attention kernels: PTX wrappers, the bounded mbarrier wait, the stream-K
+// tile cursor, the draft-tree ancestor masks and the TMA producer warp.
+#pragma once
+
+#include "kvshot_internal.h"
+
+namespace kvshot {
+namespace dev {
+namespace {  // internal linkage: every translation unit gets its own copy
+
+// ---------------------------------------------------------------- PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void set_error(int32_t* err, int code) {
+  if (err != nullptr) atomicCAS(err, 0, code);
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+// Orders this thread's generic-proxy shared-memory accesses before later
+// async-proxy (TMA) accesses to the same memory.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(done)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
+// Every pipeline wait gives up after this long, records KVSHOT_ERR_TIMEOUT
+// and lets the kernel wind down instead of spinning forever.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int32_t* err) {
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      set_error(err, KVSHOT_ERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, err);
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+// 2-D tiled TMA load (box {64 elements, rows}) into 128B-swizzled shared memory.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar,
+                                            uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ void named_barrier_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr));
+  return v;
+}
+
+__device__ __forceinline__ void ldmatrix_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                            uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                                  uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+// D += A * B, m16n8k16, bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Byte offset, inside one K or V tile, of 16-byte chunk `ch` (0..15, i.e.
+// dims 8ch..8ch+7) of key row r.  The tile is two 64-dim halves of TK rows of
+// 128 bytes; TMA's 128-byte swizzle XORs the chunk index (mod 8) with the row
+// index (mod 8).  Every 8-row group starts on a 1024-byte boundary.
+__device__ __forceinline__ uint32_t tile_off(int r, int ch) {
+  return static_cast<uint32_t>((ch >> 3) * kHalfBytes + r * 128 + (((ch & 7) ^ (r & 7)) << 4));
+}
+
+// ------------------------------------------------------------ work plan
+
+// Clamped prefix length of cache c; out-of-range values are reported.
+__device__ __forceinline__ int clamp_len(const AttnParams& p, int c) {
+  int L = p.seq_lens[c];
+  if (L < 0 || L > p.len_bound) {
+    set_error(p.err, KVSHOT_ERR_DEVICE_BOUNDS);
+    L = L < 0 ? 0 : p.len_bound;
+  }
+  return L;
+}
+
+// s_len[c] = clamped L_c; s_base[c] = first global tile of cache c (prefix sum of
+// units x tiles per unit).  Whole block participates.  CTA 0 also publishes
+// s_base to the workspace for the merge kernel.
+__device__ void build_plan(const AttnParams& p, int* s_len, int* s_base) {
+  const int HR = p.hkv * p.row_blocks;
+  for (int c = threadIdx.x; c < p.C; c += blockDim.x) {
+    const int L = clamp_len(p, c);
+    s_len[c] = L;
+    s_base[c + 1] = ((L + kTileKeys - 1) / kTileKeys + p.draft_tiles) * HR;
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    int carry = 0;
+    for (int c0 = 0; c0 < p.C; c0 += 32) {
+      const int c = c0 + lane;
+      int v = c < p.C ? s_base[c + 1] : 0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += t;
+      }
+      if (c < p.C) s_base[c + 1] = v + carry;
+      carry += __shfl_sync(0xffffffffu, v, 31);
+    }
+    if (lane == 0) s_base[0] = 0;
+  }
+  __syncthreads();
+  if (blockIdx.x == 0)
+    for (int c = threadIdx.x; c <= p.C; c += blockDim.x) p.ws_meta[c] = s_base[c];
+}
+
+// Tiles of CTA b: [b * tpc, min(T, (b + 1) * tpc)).
+__device__ __forceinline__ int tiles_per_cta(int total, int ctas) { return (total + ctas - 1) / ctas; }
+
+struct Cursor {
+  int t, t_begin, t_end;  // global tile index and this CTA's range
+  int c, hr, lt;          // cache, KV head x row block, tile within the unit
+  int L, pt, ut;          // prefix length, prefix tiles, tiles per unit
+};
+
+__device__ __forceinline__ void cursor_load_cache(Cursor& cu, const AttnParams& p, const int* s_len) {
+  cu.L = s_len[cu.c];
+  cu.pt = (cu.L + kTileKeys - 1) / kTileKeys;
+  cu.ut = cu.pt + p.draft_tiles;
+}
+
+__device__ Cursor cursor_begin(const AttnParams& p, const int* s_len, const int* s_base) {
+  Cursor cu;
+  const int total = s_base[p.C];
+  const int tpc = tiles_per_cta(total, p.num_ctas);
+  cu.t_begin = cu.t = min(total, blockIdx.x * tpc);
+  cu.t_end = min(total, cu.t + tpc);
+  cu.c = 0;
+  cu.hr = 0;
+  cu.lt = 0;
+  cu.L = cu.pt = cu.ut = 0;
+  if (cu.t >= cu.t_end) return cu;
+  int lo = 0, hi = p.C - 1;  // last cache whose first tile is <= t
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s_base[mid] <= cu.t) lo = mid;
+    else hi = mid - 1;
+  }
+  cu.c = lo;
+  cursor_load_cache(cu, p, s_len);
+  const int rem = cu.t - s_base[lo];
+  cu.hr = rem / cu.ut;
+  cu.lt = rem - cu.hr * cu.ut;
+  return cu;
+}
+
+__device__ __forceinline__ void cursor_next(Cursor& cu, const AttnParams& p, const int* s_len) {
+  ++cu.t;
+  if (++cu.lt == cu.ut) {
+    cu.lt = 0;
+    if (++cu.hr == p.hkv * p.row_blocks) {
+      cu.hr = 0;
+      ++cu.c;
+      if (cu.t < cu.t_end) cursor_load_cache(cu, p, s_len);
+    }
+  }
+}
+
+struct TileInfo {
+  bool draft;   // draft tile (else prefix tile)
+  int key0;     // first key: prefix token index, or draft slot
+  int nkeys;    // valid keys in the tile (1..TK)
+  bool first;   // first tile of this CTA's piece of the unit
+  bool last;    // last tile of this CTA's piece of the unit
+};
+
+__device__ __forceinline__ TileInfo tile_info(const Cursor& cu, const AttnParams& p) {
+  TileInfo ti;
+  ti.draft = cu.lt >= cu.pt;
+  ti.key0 = (ti.draft ? cu.lt - cu.pt : cu.lt) * kTileKeys;
+  ti.nkeys = min(kTileKeys, (ti.draft ? p.N : cu.L) - ti.key0);
+  ti.first = (cu.t == cu.t_begin) || cu.lt == 0;
+  ti.last = (cu.t == cu.t_end - 1) || cu.lt == cu.ut - 1;
+  return ti;
+}
+
+// ------------------------------------------------------ draft-tree masks
+
+// s_anc[nl] = bitmask of draft slots visible to query node N - Nq + nl: the
+// node itself and its ancestors (tree verification mask).  Built by the
+// `nthreads` consumer threads (tid in [0, nthreads)), which must all call it;
+// two named barriers (id `bar`) fence it.  Invalid parents are reported and
+// treated as roots.
+__device__ void build_ancestor_masks(const AttnParams& p, int seq, uint64_t* s_anc, int* s_par, int tid,
+                                     int nthreads, int bar) {
+  const int* par = p.tree_parent + static_cast<size_t>(seq) * p.N;
+  for (int i = tid; i < p.N; i += nthreads) {
+    int v = par[i];
+    if (v < -1 || v >= i) {
+      set_error(p.err, KVSHOT_ERR_TREE);
+      v = -1;
+    }
+    s_par[i] = v;
+  }
+  named_barrier_sync(bar, nthreads);
+  for (int nl = tid; nl < p.Nq; nl += nthreads) {
+    uint64_t bits = 0;
+    for (int m = p.N - p.Nq + nl; m >= 0; m = s_par[m]) bits |= 1ull << m;  // parents strictly decrease
+    s_anc[nl] = bits;
+  }
+  named_barrier_sync(bar, nthreads);
+}
+
+// Is draft slot m visible to query row r (row of the unit's GQA stack)?
+__device__ __forceinline__ bool draft_visible(const AttnParams& p, const uint64_t* s_anc, int r, int m) {
+  if (m >= p.N) return false;
+  const int nl = min(r / p.G, p.Nq - 1);
+  if (p.tree) return (s_anc[nl] >> m) & 1ull;
+  return m <= p.N - p.Nq + nl;
+}
+
+// ------------------------------------------------------------ TMA producer
+
+// Page id of page index `pg` of cache c (validated against the pool).
+__device__ __forceinline__ int load_page_id(const AttnParams& p, int c, int pg) {
+  int pid = p.page_table[static_cast<size_t>(c) * p.max_pages + pg];
+  if (pid < 0 || pid >= p.num_pages) {
+    set_error(p.err, KVSHOT_ERR_DEVICE_BOUNDS);
+    pid = 0;
+  }
+  return pid;
+}
+
+// Lane-distributed page ids of a paged prefix tile (lane i holds box i's page).
+__device__ __forceinline__ int tile_page_ids(const AttnParams& p, const Cursor& cu, int lane) {
+  if (cu.t >= cu.t_end || !p.paged || cu.lt >= cu.pt) return 0;
+  const int key0 = cu.lt * kTileKeys;
+  const int nkeys = min(kTileKeys, cu.L - key0);
+  const int nbox = (nkeys + p.box_rows - 1) / p.box_rows;
+  if (lane >= nbox) return 0;
+  return load_page_id(p, cu.c, (key0 + lane * p.box_rows) / p.page_size);
+}
+
+struct Pipe {
+  uint8_t* ring;       // stages x kStageBytes, 1024-aligned
+  uint64_t* full;      // [stages] TMA -> consumers
+  uint64_t* empty;     // [stages] consumers -> TMA
+  int stages;
+  volatile int* abort; // set when a wait timed out
+  int* issued;         // tiles issued by the producer
+};
+
+// The producer warp: walks this CTA's tiles and issues their TMA loads into the
+// stage ring, one tile ahead on the page-table reads.  Lane 0 issues.
+__device__ void run_producer(const AttnParams& p, const TensorMaps& maps, const Pipe& pipe, const int* s_len,
+                             Cursor cu) {
+  const int lane = threadIdx.x & 31;
+  const uint64_t policy = l2_policy_evict_first();
+  int stage = 0;
+  uint32_t phase = 0;
+  int issued = 0;
+  int pid_cur = tile_page_ids(p, cu, lane);
+  while (cu.t < cu.t_end) {
+    Cursor nx = cu;
+    cursor_next(nx, p, s_len);
+    const int pid_next = tile_page_ids(p, nx, lane);  // in flight while we wait for a free stage
+
+    const int h = cu.hr / p.row_blocks;
+    const int L = cu.L;
+    const bool draft = cu.lt >= cu.pt;
+    const int key0 = (draft ? cu.lt - cu.pt : cu.lt) * kTileKeys;
+    const int nkeys = min(kTileKeys, (draft ? p.N : L) - key0);
+    // Lane-distributed ids -> lane 0 (shuffles are warp-wide).
+    int pids[kTileKeys / 8];
+#pragma unroll
+    for (int i = 0; i < kTileKeys / 8; ++i) pids[i] = __shfl_sync(0xffffffffu, pid_cur, i);
+
+    int ok = 1;
+    if (lane == 0) {
+      ok = mbar_wait(smem_addr(&pipe.empty[stage]), phase ^ 1u, p.err) ? 1 : 0;
+      if (!ok || *pipe.abort) ok = 0;
+    }
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (!ok) {
+      if (lane == 0) *pipe.abort = 1;
+      break;
+    }
+    if (lane == 0) {
+      const uint32_t full_bar = smem_addr(&pipe.full[stage]);
+      const uint32_t kdst = smem_addr(pipe.ring + static_cast<size_t>(stage) * kStageBytes);
+      const uint32_t vdst = kdst + kKVTileBytes;
+      if (draft) {
+        const int nbox = (nkeys + kDraftBoxRows - 1) / kDraftBoxRows;
+        mbar_arrive_expect_tx(full_bar, nbox * kDraftBoxRows * 128 * 4);
+        const int y0 = (cu.c * p.hkv + h) * p.n_max + key0;
+        for (int i = 0; i < nbox; ++i) {
+          const uint32_t off = i * kDraftBoxRows * 128;
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf) {
+            tma_load_2d(kdst + hf * kHalfBytes + off, &maps.dk, hf * 64, y0 + i * kDraftBoxRows, full_bar, policy);
+            tma_load_2d(vdst + hf * kHalfBytes + off, &maps.dv, hf * 64, y0 + i * kDraftBoxRows, full_bar, policy);
+          }
+        }
+      } else if (p.paged) {
+        const int br = p.box_rows;
+        const int nbox = (nkeys + br - 1) / br;
+        mbar_arrive_expect_tx(full_bar, nbox * br * 128 * 4);
+#pragma unroll
+        for (int i = 0; i < kTileKeys / 8; ++i) {  // box_rows >= 8, so at most 8 boxes
+          if (i < nbox) {
+            const int krow = key0 + i * br;
+            const int y = (pids[i] * p.hkv + h) * p.page_size + (krow % p.page_size);
+            const uint32_t off = i * br * 128;
+#pragma unroll
+            for (int hf = 0; hf < 2; ++hf) {
+              tma_load_2d(kdst + hf * kHalfBytes + off, &maps.tk, hf * 64, y, full_bar, policy);
+              tma_load_2d(vdst + hf * kHalfBytes + off, &maps.tv, hf * 64, y, full_bar, policy);
+            }
+          }
+        }
+      } else {
+        mbar_arrive_expect_tx(full_bar, kTileKeys * 128 * 4);
+        const int y = (cu.c * p.hkv + h) * p.l_cap + key0;
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+          tma_load_2d(kdst + hf * kHalfBytes, &maps.tk, hf * 64, y, full_bar, policy);
+          tma_load_2d(vdst + hf * kHalfBytes, &maps.tv, hf * 64, y, full_bar, policy);
+        }
+      }
+    }
+    ++issued;
+    pid_cur = pid_next;
+    cu = nx;
+    if (++stage == pipe.stages) {
+      stage = 0;
+      phase ^= 1u;
+    }
+  }
+  if (lane == 0) *pipe.issued = issued;
+}
+
+// After the roles finish: if a wait timed out, wait (bounded) for every TMA
+// load still in flight so no copy lands in shared memory after the CTA exits.
+// Called by one thread after a block-wide barrier.
+__device__ void drain_after_abort(const AttnParams& p, const Pipe& pipe, int consumed) {
+  if (!*pipe.abort) return;
+  for (int k = consumed; k < *pipe.issued; ++k) {
+    const int st = k % pipe.stages;
+    const uint32_t par = static_cast<uint32_t>((k / pipe.stages) & 1);
+    if (!mbar_wait(smem_addr(&pipe.full[st]), par, p.err)) break;
+  }
+}
+
+}  // namespace
+}  // namespace dev
+}  // namespace kvshot

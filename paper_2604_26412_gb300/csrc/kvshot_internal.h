@@ -1,0 +1,88 @@
+// kvshot_internal.h -- declarations shared by libkvshot's translation units.
+//
+// Work decomposition of kvshot_draft_attn (see kvshot_attn_common.cuh):
+//   unit  = (cache c, KV head h, row block rb): the stacked query rows of one
+//           GQA group (G heads x Nq draft nodes, or a 64-row block of them).
+//           Every unit streams the same keys: L_c prefix tokens then the N
+//           draft slots.
+//   tile  = TK consecutive keys of one unit (prefix tiles first, then draft
+//           tiles), staged into shared memory by TMA as one K and one V block.
+//   The tiles of all units are laid end to end (cache-major) and cut into
+//   equal contiguous ranges, one per persistent CTA ("stream-K" split), so
+//   ragged prefix lengths stay balanced.  A unit whose tiles straddle CTAs is
+//   computed as pieces whose softmax states are merged afterwards.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "kvshot.h"
+
+namespace kvshot {
+
+constexpr int kHeadDim = 128;
+constexpr int kTileKeys = 64;                         // TK
+constexpr int kHalfBytes = kTileKeys * 128;           // 64 dims x TK keys, bf16: one TMA-swizzled half
+constexpr int kKVTileBytes = 2 * kHalfBytes;          // one K (or V) tile
+constexpr int kStageBytes = 2 * kKVTileBytes;         // K + V
+constexpr int kMaxCaches = 1024;
+constexpr int kMaxTreeNodes = 64;
+constexpr int kDraftBoxRows = 8;                      // draft K/V are loaded 8 rows per TMA box
+constexpr int kCcRows = 4;                            // rows per unit of the CUDA-core kernel
+constexpr int kMmaMaxTiles = 4;                       // m16 tiles per unit of the tensor-core kernel
+
+// Everything a draft-attention kernel needs besides the tensor maps.
+struct AttnParams {
+  const __nv_bfloat16* q;
+  __nv_bfloat16* out;
+  float* lse;
+  const int32_t* page_table;
+  const int32_t* seq_lens;
+  const int32_t* tree_parent;
+  int32_t* err;             // may be null
+  int32_t* ws_meta;         // [C + 1] tile prefix per cache, written by CTA 0
+  float* ws_lse;            // [slots, rows_per_unit] log2-domain lse of pieces
+  float* ws_o;              // [slots, rows_per_unit, 128] normalised piece outputs
+  int C, B, hq, hkv, G;
+  int rows_total;           // G * Nq
+  int rows_per_unit;        // rows of one unit (<= rows_total)
+  int row_blocks;           // RB = ceil(rows_total / rows_per_unit)
+  int paged, page_size, max_pages, num_pages, l_cap;
+  int box_rows;             // rows per target TMA box: min(page_size, TK) paged, TK contiguous
+  int len_bound;            // min(max_seq_len, capacity): seq_lens are clamped to [0, len_bound]
+  int N, Nq, n_max, tree;
+  int draft_tiles;          // ceil(N / TK)
+  float qscale;             // softmax scale * log2(e): scores are kept in the log2 domain
+  int num_ctas;             // persistent grid size
+};
+
+struct AppendParams {
+  const __nv_bfloat16* q_in;
+  const __nv_bfloat16* k_in;
+  const __nv_bfloat16* v_in;
+  const int32_t* positions;
+  __nv_bfloat16* draft_k;
+  __nv_bfloat16* draft_v;
+  __nv_bfloat16* q_out;
+  int C, hq, hkv, n_max, n0, n_new;
+  double inv_freq[kHeadDim / 2];  // rope_base^(-2j/128) in fp64
+};
+
+struct TensorMaps {
+  CUtensorMap tk, tv, dk, dv;
+};
+
+// Kernel launchers (one per translation unit).  Return cudaSuccess or the launch error.
+cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, cudaStream_t stream);
+cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, cudaStream_t stream);
+cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream);
+cudaError_t launch_append(const AppendParams& a, cudaStream_t stream);
+
+// CTAs per SM each kernel variant is built for (its shared-memory ring and
+// register budget are sized for this residency).
+int attn_cc_ctas_per_sm();
+int attn_mma_ctas_per_sm(int m_tiles);
+
+}  // namespace kvshot

@@ -1,0 +1,138 @@
+"""The C ABI boundary, on the CPU: the library builds, loads and exports every
+function include/kvshot.h declares; the Python descriptor mirrors the C
+struct byte for byte; invalid arguments are rejected with their status code
+before anything touches CUDA."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2604_26412_gb300 import build as kbuild
+from paper_2604_26412_gb300 import kvshot
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "kvshot.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    kbuild.build()
+    return kvshot.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(kvshot_\w+)\s*\(", text)))
+
+
+def test_header_functions_are_exported(lib):
+    names = declared_functions()
+    assert set(names) == set(kvshot.EXPORTS)
+    out = subprocess.run(["nm", "-D", "--defined-only", kbuild.LIB], capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (kvshot_\w+)", out))
+    for n in names:
+        assert n in exported, n
+        assert hasattr(lib, n)
+
+
+def test_descriptor_layout_matches_header(tmp_path):
+    fields = [f for f, _ in kvshot.AttnDesc._fields_]
+    src = ["#include <stdio.h>", "#include <stddef.h>", '#include "kvshot.h"', "int main(void) {",
+           'printf("%zu\\n", sizeof(kvshot_attn_desc));']
+    src += [f'printf("%zu\\n", offsetof(kvshot_attn_desc, {f}));' for f in fields]
+    src += ["return 0; }"]
+    c = tmp_path / "layout.c"
+    c.write_text("\n".join(src))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.dirname(HEADER), str(c), "-o", str(exe)], check=True)
+    vals = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    assert vals[0] == ctypes.sizeof(kvshot.AttnDesc)
+    for f, off in zip(fields, vals[1:]):
+        assert getattr(kvshot.AttnDesc, f).offset == off, f
+
+
+def test_status_strings_and_version(lib):
+    for code in range(0, 10):
+        assert kvshot.status_string(code) and kvshot.status_string(code) != "unknown status"
+    assert kvshot.status_string(42) == "unknown status"
+    assert kvshot.version() >= 100
+
+
+def _desc(**kw):
+    base = dict(num_caches=2, num_seqs=2, hq=32, hkv=8, n_nodes=8, n_query=4, n_max=8, max_seq_len=64,
+                page_size=16, max_pages_per_seq=4, num_pages=8, l_cap=64, tree=True)
+    base.update(kw)
+    return kvshot.make_desc(**base)
+
+
+# Fake, suitably aligned device addresses: never dereferenced, because every
+# case below fails validation first.
+A = 1 << 20
+
+
+def _attn(d, **ptrs):
+    p = dict(q=A, tk=A, tv=A, pt=A, sl=A, dk=A, dv=A, par=A, out=2 * A, lse=3 * A)
+    p.update(ptrs)
+    return kvshot.draft_attn_status(d, p["q"], p["tk"], p["tv"], p["pt"], p["sl"], p["dk"], p["dv"], p["par"], p["out"],
+                                    p["lse"], stream=0)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(num_caches=0), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(num_caches=3, num_seqs=2), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(num_caches=2048, num_seqs=2048), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    (dict(hq=30, hkv=8), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(head_dim=64), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    (dict(n_query=9), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(n_nodes=9), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(n_nodes=65, n_max=80), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    (dict(page_size=12), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    (dict(page_size=512), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    (dict(page_size=24), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    (dict(page_size=72), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    (dict(num_pages=0), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(max_seq_len=-1), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(flags=0x80), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(flags=kvshot.KVSHOT_FORCE_CC | kvshot.KVSHOT_FORCE_MMA), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(num_ctas=-1), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(scale=float("inf")), kvshot.KVSHOT_ERR_SHAPE),
+])
+def test_invalid_descriptor_codes(lib, kw, code):
+    assert _attn(_desc(**kw)) == code
+    if "page_size" not in kw and "num_pages" not in kw:
+        assert kvshot.workspace_size(_desc(**kw)) == 0
+
+
+def test_null_and_alignment_codes(lib):
+    assert kvshot.draft_attn_status(None, A, A, A, A, A, A, A, A, A, A, stream=0) == kvshot.KVSHOT_ERR_NULL
+    d = _desc()
+    assert _attn(d, q=None) == kvshot.KVSHOT_ERR_NULL
+    assert _attn(d, par=None) == kvshot.KVSHOT_ERR_NULL        # tree needs parents
+    assert _attn(d, sl=None) == kvshot.KVSHOT_ERR_NULL
+    assert _attn(d, q=A + 8) == kvshot.KVSHOT_ERR_ALIGN
+    assert _attn(d, tk=A + 2) == kvshot.KVSHOT_ERR_ALIGN
+    assert _attn(d, lse=A + 2) == kvshot.KVSHOT_ERR_ALIGN
+    assert _attn(d, out=A + 4) == kvshot.KVSHOT_ERR_ALIGN
+    assert _attn(_desc(l_cap=0), pt=None) == kvshot.KVSHOT_ERR_SHAPE   # contiguous layout needs l_cap
+    assert _attn(_desc(n_query=0)) == kvshot.KVSHOT_OK                  # no-op
+
+
+def test_append_argument_codes(lib):
+    d = _desc()
+    call = lambda **k: kvshot.draft_append_status(d, k.get("q", A), k.get("k", A), k.get("v", A), k.get("pos", A),
+                                                  k.get("n0", 0), k.get("n_new", 2), k.get("base", 1e6), A, A,
+                                                  k.get("qo", 2 * A), stream=0)
+    assert kvshot.draft_append_status(None, A, A, A, A, 0, 1, 1e6, A, A, A, stream=0) == kvshot.KVSHOT_ERR_NULL
+    assert call(n0=7, n_new=2) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(n0=-1) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(base=0.0) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(n_new=0) == kvshot.KVSHOT_OK
+    assert call(q=None) == kvshot.KVSHOT_ERR_NULL
+    assert call(k=A + 4) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(pos=A + 2) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(qo=A + 256) == kvshot.KVSHOT_ERR_SHAPE                 # partial overlap of q_out and q_in
+    assert kvshot.draft_append_status(_desc(head_dim=96), A, A, A, A, 0, 1, 1e6, A, A, A, stream=0) == \
+        kvshot.KVSHOT_ERR_UNSUPPORTED
