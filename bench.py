@@ -58,6 +58,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seconds", type=float, default=12.0)
     ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--page-size", type=int, default=0,
+                    help="override the workload's page size (exploration; the default is the workload's own)")
     return ap.parse_args()
 
 
@@ -274,6 +276,8 @@ def run_ours(args, world, rank, local):
 
     dev = torch.device("cuda", torch.cuda.current_device())
     spec = wl.config(args.workload, seed=args.seed)
+    if args.page_size:
+        spec.page_size = args.page_size
     inp = wl.make_inputs(spec, dev, seed=args.seed + 1000 * rank)
     flags = {"auto": 0, "cc": kvshot.KVSHOT_FORCE_CC, "mma": kvshot.KVSHOT_FORCE_MMA}[args.kernel]
     step = DraftStep(inp, mode=args.mode, flags=flags, num_ctas=args.num_ctas)

@@ -50,7 +50,7 @@ __host__ __device__ inline size_t smem_bytes(int C) {
   size_t off = static_cast<size_t>(CF::kStages) * kStageBytes;
   off += 2 * CF::kStages * sizeof(uint64_t);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
-  off += sizeof(float) * CF::kMT * 16 * kCombStride;
+  if (CF::kKS > 1) off += sizeof(float) * CF::kMT * 16 * kCombStride;  // only slices > 1 combine through smem
   off += 2 * sizeof(float) * CF::kKS * CF::kRows;
   off += sizeof(int) * 4;
   off += sizeof(int) * (2 * C + 1);
@@ -68,7 +68,7 @@ __device__ Smem carve(uint8_t* raw, int C) {
   s.anc = s.empty + CF::kStages;
   s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
   s.comb_o = reinterpret_cast<float*>(s.par + kMaxTreeNodes);
-  s.comb_m = s.comb_o + CF::kMT * 16 * kCombStride;
+  s.comb_m = s.comb_o + (CF::kKS > 1 ? CF::kMT * 16 * kCombStride : 0);
   s.comb_l = s.comb_m + CF::kKS * CF::kRows;
   s.misc = reinterpret_cast<int*>(s.comb_l + CF::kKS * CF::kRows);
   s.len = s.misc + 4;

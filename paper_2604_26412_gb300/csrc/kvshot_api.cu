@@ -115,7 +115,13 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   const int G = d->hq / d->hkv;
   const int rows = G * d->n_query;
   const bool force_cc = d->flags & KVSHOT_FORCE_CC, force_mma = d->flags & KVSHOT_FORCE_MMA;
-  pl->mma = force_mma || (!force_cc && rows > kCcRows);
+  // Measured on GB300 (ncu + bench): at 4 stacked rows the CUDA-core kernel is
+  // issue/latency bound (IPC ~1, ~100 warp instructions per key) while the
+  // m16n8k16 kernel, with the stack zero-padded to 16 rows, streams K/V at
+  // 73-97% of HBM bandwidth; so the tensor-core kernel is the default for every
+  // stack size and the CUDA-core kernel is kept behind KVSHOT_FORCE_CC.
+  (void)force_mma;
+  pl->mma = !force_cc;
   if (pl->mma) {
     pl->m_tiles = std::min(kMmaMaxTiles, std::max(1, (rows + 15) / 16));
     pl->rows_per_unit = 16 * pl->m_tiles;

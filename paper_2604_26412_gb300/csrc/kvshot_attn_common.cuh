@@ -308,24 +308,25 @@ __device__ __forceinline__ bool draft_visible(const AttnParams& p, const uint64_
 
 // ------------------------------------------------------------ TMA producer
 
-// Page id of page index `pg` of cache c (validated against the pool).
-__device__ __forceinline__ int load_page_id(const AttnParams& p, int c, int pg) {
-  int pid = p.page_table[static_cast<size_t>(c) * p.max_pages + pg];
-  if (pid < 0 || pid >= p.num_pages) {
-    set_error(p.err, KVSHOT_ERR_DEVICE_BOUNDS);
-    pid = 0;
-  }
-  return pid;
-}
-
-// Lane-distributed page ids of a paged prefix tile (lane i holds box i's page).
+// Raw (unvalidated) lane-distributed page ids of a paged prefix tile: lane i
+// holds box i's page.  Validation happens at use time (valid_page_id), so the
+// load stays in flight while the producer waits for a free stage.
 __device__ __forceinline__ int tile_page_ids(const AttnParams& p, const Cursor& cu, int lane) {
   if (cu.t >= cu.t_end || !p.paged || cu.lt >= cu.pt) return 0;
   const int key0 = cu.lt * kTileKeys;
   const int nkeys = min(kTileKeys, cu.L - key0);
   const int nbox = (nkeys + p.box_rows - 1) / p.box_rows;
   if (lane >= nbox) return 0;
-  return load_page_id(p, cu.c, (key0 + lane * p.box_rows) / p.page_size);
+  return p.page_table[static_cast<size_t>(cu.c) * p.max_pages + (key0 + lane * p.box_rows) / p.page_size];
+}
+
+// A page id checked against the pool; out-of-range ids are reported and replaced by page 0.
+__device__ __forceinline__ int valid_page_id(const AttnParams& p, int pid) {
+  if (pid < 0 || pid >= p.num_pages) {
+    set_error(p.err, KVSHOT_ERR_DEVICE_BOUNDS);
+    pid = 0;
+  }
+  return pid;
 }
 
 struct Pipe {
@@ -359,6 +360,7 @@ __device__ void run_producer(const AttnParams& p, const TensorMaps& maps, const 
     const int nkeys = min(kTileKeys, (draft ? p.N : L) - key0);
     // Lane-distributed ids -> lane 0 (shuffles are warp-wide).
     int pids[kTileKeys / 8];
+    if (p.paged && !draft) pid_cur = valid_page_id(p, pid_cur);
 #pragma unroll
     for (int i = 0; i < kTileKeys / 8; ++i) pids[i] = __shfl_sync(0xffffffffu, pid_cur, i);
 

@@ -166,7 +166,7 @@ def test_device_errors_are_reported_without_fault():
         _run(spec, inp, dk, dv, q, N, Nq)
     inp.seq_lens[0] = 100
     # a parent that is not an earlier node
-    par = inp.tree_parent[:, :N].contiguous()
+    par = inp.tree_parent[:, :N].clone()
     par[0, 3] = 3
     with pytest.raises(AssertionError, match="device error 5"):
         _run(spec, inp, dk, dv, q, N, Nq, parents=par)
