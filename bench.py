@@ -37,6 +37,7 @@ import torch
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+from paper_2604_26412_gb300 import replicas  # noqa: E402
 from paper_2604_26412_gb300 import workloads as wl  # noqa: E402
 
 METRIC = "draft-attn tokens/s and achieved HBM GB/s (fraction of GB300 peak) at 1 GPU"
@@ -58,6 +59,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seconds", type=float, default=12.0)
     ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--max-prefix", type=int, default=0,
+                    help="cap every prefix length (profiling-sized cases; the default is the workload's own)")
     ap.add_argument("--page-size", type=int, default=0,
                     help="override the workload's page size (exploration; the default is the workload's own)")
     return ap.parse_args()
@@ -79,18 +82,11 @@ def dist_setup():
 
 
 def barrier(world):
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
+    replicas.barrier()
 
 
 def max_over_ranks(x: float, world: int) -> float:
-    if world == 1:
-        return x
-    import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
+    return replicas.max_over_ranks(x)
 
 
 def measured_peaks():
@@ -278,6 +274,8 @@ def run_ours(args, world, rank, local):
     spec = wl.config(args.workload, seed=args.seed)
     if args.page_size:
         spec.page_size = args.page_size
+    if args.max_prefix:
+        spec.seq_lens = [min(L, args.max_prefix) for L in spec.seq_lens]
     inp = wl.make_inputs(spec, dev, seed=args.seed + 1000 * rank)
     flags = {"auto": 0, "cc": kvshot.KVSHOT_FORCE_CC, "mma": kvshot.KVSHOT_FORCE_MMA}[args.kernel]
     step = DraftStep(inp, mode=args.mode, flags=flags, num_ctas=args.num_ctas)
@@ -323,7 +321,7 @@ def run_ours(args, world, rank, local):
     ms_total = max_over_ranks(t_start.elapsed_time(t_end), world)
     ms_per_step = ms_total / args.steps
     tokens_per_step = step.tokens
-    value = tokens_per_step * world * args.steps / (ms_total / 1e3)
+    value = replicas.whole_job_rate(tokens_per_step, args.steps, world, ms_total)
 
     # ---- live roofline of the draft-attention call (attention + merge kernels), per level
     levels = step.levels
@@ -447,7 +445,7 @@ def run_e2e(args, step, inp, stream, world):
         b.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(a.elapsed_time(b), world)
-    value = step.tokens * world * steps / (ms / 1e3)
+    value = replicas.whole_job_rate(step.tokens, steps, world, ms)
     return {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "steps": steps, "api": "kvshot_draft_append + kvshot_draft_attn via ctypes, no CUDA graph"}
 
