@@ -130,6 +130,37 @@ kvshot_status kvshot_draft_attn(const kvshot_attn_desc* desc, const void* q, con
                                 const void* draft_k, const void* draft_v, const int32_t* tree_parent,
                                 void* out, float* lse, kvshot_stream_t stream);
 
+/* Bytes of device scratch built into the library for kvshot_draft_attn_static (32 MiB). */
+#define KVSHOT_STATIC_WORKSPACE_BYTES (32u * 1024u * 1024u)
+
+/*
+ * kvshot_draft_attn_static -- the same computation, arguments and results as
+ * kvshot_draft_attn, for callers that cannot allocate device memory: code
+ * handed only device pointers by a host framework that owns all allocation,
+ * a serving loop whose memory pool is fully reserved up front, or a hot path
+ * that must not call cudaMalloc (which can synchronise the device and stall
+ * every other stream).  The paper has no counterpart; this is an interface
+ * convenience only.
+ *
+ * Instead of desc->workspace (ignored, as is desc->workspace_bytes) the call
+ * uses a fixed scratch array of KVSHOT_STATIC_WORKSPACE_BYTES inside the
+ * library; every GPU that loads the library holds that array until the
+ * process exits.  The call itself allocates nothing.
+ *  - Descriptors whose work plan needs more scratch than that
+ *    (kvshot_draft_attn_workspace_size(desc) > KVSHOT_STATIC_WORKSPACE_BYTES)
+ *    are rejected with KVSHOT_ERR_WORKSPACE before anything is launched.
+ *  - The first call on each device looks up the array's device address (with
+ *    that device current); make that first call before any stream capture.
+ *  - All calls on a device share the one array and it keeps the last call's
+ *    contents.  Nothing in it has to start at zero, but two calls whose
+ *    kernels overlap on the GPU (e.g. on different streams without ordering)
+ *    race on it and corrupt each other's results; keep such calls ordered.
+ */
+kvshot_status kvshot_draft_attn_static(const kvshot_attn_desc* desc, const void* q, const void* target_k,
+                                       const void* target_v, const int32_t* page_table, const int32_t* seq_lens,
+                                       const void* draft_k, const void* draft_v, const int32_t* tree_parent,
+                                       void* out, float* lse, kvshot_stream_t stream);
+
 /*
  * Draft append with RoPE: the drafter's new K/V for draft positions j > t
  * enter M_i (App. B: "the drafter generates its own KV via learned

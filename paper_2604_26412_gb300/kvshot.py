@@ -32,7 +32,8 @@ KVSHOT_FORCE_CC = 0x2
 KVSHOT_FORCE_MMA = 0x4
 
 EXPORTS = ("kvshot_draft_attn", "kvshot_draft_attn_workspace_size", "kvshot_draft_append", "kvshot_status_string",
-           "kvshot_version")
+           "kvshot_version", "kvshot_draft_attn_static")
+STATIC_WORKSPACE_BYTES = 32 * 1024 * 1024  # KVSHOT_STATIC_WORKSPACE_BYTES
 
 
 class KvshotError(RuntimeError):
@@ -88,6 +89,8 @@ def load(build_if_missing: bool = True):
     P = ctypes.c_void_p
     lib.kvshot_draft_attn.argtypes = [ctypes.POINTER(AttnDesc), P, P, P, P, P, P, P, P, P, P, P]
     lib.kvshot_draft_attn.restype = ctypes.c_int
+    lib.kvshot_draft_attn_static.argtypes = [ctypes.POINTER(AttnDesc), P, P, P, P, P, P, P, P, P, P, P]
+    lib.kvshot_draft_attn_static.restype = ctypes.c_int
     lib.kvshot_draft_attn_workspace_size.argtypes = [ctypes.POINTER(AttnDesc)]
     lib.kvshot_draft_attn_workspace_size.restype = ctypes.c_size_t
     lib.kvshot_draft_append.argtypes = [ctypes.POINTER(AttnDesc), P, P, P, P, ctypes.c_int32, ctypes.c_int32,
@@ -158,6 +161,14 @@ def draft_attn(desc: AttnDesc, q, target_k, target_v, page_table, seq_lens, draf
                            lse, stream)
     if st != KVSHOT_OK:
         raise KvshotError(st, "kvshot_draft_attn")
+
+
+def draft_attn_static_status(desc: AttnDesc, q, target_k, target_v, page_table, seq_lens, draft_k, draft_v,
+                             tree_parent, out, lse, stream=None) -> int:
+    """Call kvshot_draft_attn_static (library-owned scratch, no allocation) and return its status."""
+    return int(load().kvshot_draft_attn_static(_dref(desc), _ptr(q), _ptr(target_k), _ptr(target_v),
+                                               _ptr(page_table), _ptr(seq_lens), _ptr(draft_k), _ptr(draft_v),
+                                               _ptr(tree_parent), _ptr(out), _ptr(lse), _stream(stream)))
 
 
 def draft_append_status(desc: AttnDesc, q_in, k_in, v_in, positions, n0: int, n_new: int, rope_base: float, draft_k,
