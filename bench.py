@@ -53,7 +53,7 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", type=int, default=5, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--mode", choices=["per_depth", "whole"], default="per_depth")
-    ap.add_argument("--kernel", choices=["auto", "cc", "mma"], default="auto")
+    ap.add_argument("--kernel", choices=["auto", "cc", "mma", "tc"], default="auto")
     ap.add_argument("--num-ctas", type=int, default=0)
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -277,7 +277,8 @@ def run_ours(args, world, rank, local):
     if args.max_prefix:
         spec.seq_lens = [min(L, args.max_prefix) for L in spec.seq_lens]
     inp = wl.make_inputs(spec, dev, seed=args.seed + 1000 * rank)
-    flags = {"auto": 0, "cc": kvshot.KVSHOT_FORCE_CC, "mma": kvshot.KVSHOT_FORCE_MMA}[args.kernel]
+    flags = {"auto": 0, "cc": kvshot.KVSHOT_FORCE_CC, "mma": kvshot.KVSHOT_FORCE_MMA,
+             "tc": kvshot.KVSHOT_FORCE_TC}[args.kernel]
     step = DraftStep(inp, mode=args.mode, flags=flags, num_ctas=args.num_ctas)
     paged = inp.page_table is not None
     stream = torch.cuda.Stream()

@@ -59,7 +59,8 @@ typedef enum kvshot_status {
 /* desc->flags */
 #define KVSHOT_TREE 0x1u       /* draft nodes form a tree given by tree_parent (else a chain) */
 #define KVSHOT_FORCE_CC 0x2u   /* use the CUDA-core kernel whatever the row count (measurement aid) */
-#define KVSHOT_FORCE_MMA 0x4u  /* use the tensor-core kernel whatever the row count (measurement aid) */
+#define KVSHOT_FORCE_MMA 0x4u  /* use the mma.sync tensor-core kernel whatever the row count (measurement aid) */
+#define KVSHOT_FORCE_TC 0x8u   /* use the tcgen05 / tensor-memory kernel (needs 128 % (hq / hkv) == 0) */
 
 /*
  * Problem descriptor shared by kvshot_draft_attn and kvshot_draft_append.
@@ -84,7 +85,7 @@ typedef struct kvshot_attn_desc {
   int32_t n_query;           /* Nq: the last Nq draft nodes are the query rows (Nq <= N) */
   int32_t n_max;             /* draft buffer capacity in slots (N <= n_max) */
   float scale;               /* softmax scale on q.k; 0 selects 1/sqrt(head_dim) */
-  uint32_t flags;            /* KVSHOT_TREE, KVSHOT_FORCE_CC, KVSHOT_FORCE_MMA */
+  uint32_t flags;            /* KVSHOT_TREE, at most one of KVSHOT_FORCE_CC / _MMA / _TC */
   int32_t num_ctas;          /* persistent CTAs to launch; 0 = one full wave on this GPU */
   void* workspace;           /* device scratch, 256-byte aligned; see kvshot_draft_attn_workspace_size */
   size_t workspace_bytes;

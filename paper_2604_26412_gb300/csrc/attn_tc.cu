@@ -1,0 +1,527 @@
+// attn_tc.cu -- draft attention on the 5th-generation tensor cores (tcgen05),
+// accumulators in tensor memory (TMEM).
+//
+// Per unit (cache, KV head, block of up to 128 stacked GQA rows), per 64-key
+// tile (Sec. 2.2 Eq. "kv-reattention" over the memory M_i of Sec. 3.4 /
+// App. B, as an online softmax in the log2 domain):
+//   S = Q K^T      tcgen05.mma M=128 N=64  K=128 (8 x K16), A = Q (smem), B = K tile (smem), D = S (TMEM)
+//   P = softmax(S) one thread per row: TMEM -> registers -> bf16 P (smem, 128B-swizzled)
+//   O += P V       tcgen05.mma M=128 N=128 K=64 (4 x K16), A = P (smem), B = V tile (smem, MN-major), D = O (TMEM)
+// Warp roles: warp 0 issues TMA (K/V tiles, one q block per piece), warp 1
+// owns TMEM and one of its threads issues every MMA, warps 2..5 run the
+// softmax and the epilogue (thread = TMEM lane = row).  S is double-buffered
+// in TMEM so QK^T of tile t+1 overlaps the softmax of tile t; O is rescaled in
+// TMEM only when a row's running max grows by more than 2^8 (lazy rescale).
+// Rows of the 128-row MMA beyond the unit's stack carry no output.
+#include "kvshot_attn_common.cuh"
+
+namespace kvshot {
+namespace {
+
+using namespace dev;
+
+constexpr int kStages = 3;
+constexpr int kThreads = 6 * 32;
+constexpr int kSoftmaxThreads = 128;
+constexpr int kBarSoftmax = 1;             // named barrier among the softmax warps
+constexpr int kPBufBytes = kQRows * 128;   // 128 rows x 64 keys bf16
+constexpr uint32_t kTmemCols = 256;        // S0 [0,64) S1 [64,128) O [128,256)
+constexpr uint32_t kTmemO = 128;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max grows by > 256x
+
+// ------------------------------------------------------------ tcgen05 wrappers
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred acc;\n\t"
+      "setp.ne.b32 acc, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, acc;\n\t}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrives (once) on `bar` when every tcgen05 operation this thread issued so far has completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+#define KV_R32(p) "=r"(p[0]), "=r"(p[1]), "=r"(p[2]), "=r"(p[3]), "=r"(p[4]), "=r"(p[5]), "=r"(p[6]), "=r"(p[7]), \
+    "=r"(p[8]), "=r"(p[9]), "=r"(p[10]), "=r"(p[11]), "=r"(p[12]), "=r"(p[13]), "=r"(p[14]), "=r"(p[15]),          \
+    "=r"(p[16]), "=r"(p[17]), "=r"(p[18]), "=r"(p[19]), "=r"(p[20]), "=r"(p[21]), "=r"(p[22]), "=r"(p[23]),        \
+    "=r"(p[24]), "=r"(p[25]), "=r"(p[26]), "=r"(p[27]), "=r"(p[28]), "=r"(p[29]), "=r"(p[30]), "=r"(p[31])
+#define KV_W32(p) "r"(p[0]), "r"(p[1]), "r"(p[2]), "r"(p[3]), "r"(p[4]), "r"(p[5]), "r"(p[6]), "r"(p[7]), \
+    "r"(p[8]), "r"(p[9]), "r"(p[10]), "r"(p[11]), "r"(p[12]), "r"(p[13]), "r"(p[14]), "r"(p[15]),          \
+    "r"(p[16]), "r"(p[17]), "r"(p[18]), "r"(p[19]), "r"(p[20]), "r"(p[21]), "r"(p[22]), "r"(p[23]),        \
+    "r"(p[24]), "r"(p[25]), "r"(p[26]), "r"(p[27]), "r"(p[28]), "r"(p[29]), "r"(p[30]), "r"(p[31])
+
+// 32 consecutive 32-bit TMEM columns of this warp's 32 lanes (one per thread).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : KV_R32(v)
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      KV_W32(v)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// Shared-memory matrix descriptor, 128-byte swizzle.  Start address, leading
+// and stride byte offsets are encoded >> 4; bits 46..48 hold the fixed 0b001;
+// bits 61..63 select the 128-byte swizzle (2).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= 1ull << 46;
+  d |= 2ull << 61;
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulate, bf16 A and B, A K-major,
+// B K-major (b_mn_major = false) or MN-major, shape M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+         (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+// ------------------------------------------------------------ shared memory
+
+struct Smem {
+  uint8_t* ring;       // kStages x (K tile | V tile)
+  uint8_t* qbuf;       // 2 x kQBufBytes
+  uint8_t* pbuf;       // 2 x kPBufBytes
+  uint64_t* full;      // [kStages]
+  uint64_t* empty;     // [kStages]  (MMA completion)
+  uint64_t* qfull;     // [2]
+  uint64_t* qempty;    // [2]
+  uint64_t* sfull;     // [2]  S buffer written (MMA completion)
+  uint64_t* pfull;     // [2]  P buffer written (128 softmax threads)
+  uint64_t* pvdone;    // [2]  P.V of the tile using that buffer completed
+  uint64_t* ofree;     // [1]  epilogue finished reading O
+  uint64_t* mmadone;   // [1]  every MMA completed
+  uint64_t* anc;       // [64]
+  int* par;            // [64]
+  uint32_t* tmem_base;
+  int* misc;           // [0] abort, [1] tiles issued, [2] tiles consumed, [3] q blocks issued, [4] q consumed
+  int* len;
+  int* base;
+};
+
+__host__ __device__ inline size_t smem_bytes(int C) {
+  size_t off = static_cast<size_t>(kStages) * kStageBytes + 2 * kQBufBytes + 2 * kPBufBytes;
+  off += sizeof(uint64_t) * (2 * kStages + 2 * 5 + 2);
+  off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
+  off += sizeof(uint32_t) * 4 + sizeof(int) * 8;
+  off += sizeof(int) * (2 * C + 1);
+  return off + 1024;
+}
+
+__device__ Smem carve(uint8_t* raw, int C) {
+  Smem s;
+  uint8_t* p = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
+  s.ring = p;
+  p += kStages * kStageBytes;
+  s.qbuf = p;
+  p += 2 * kQBufBytes;
+  s.pbuf = p;
+  p += 2 * kPBufBytes;
+  uint64_t* b = reinterpret_cast<uint64_t*>(p);
+  s.full = b;
+  s.empty = s.full + kStages;
+  s.qfull = s.empty + kStages;
+  s.qempty = s.qfull + 2;
+  s.sfull = s.qempty + 2;
+  s.pfull = s.sfull + 2;
+  s.pvdone = s.pfull + 2;
+  s.ofree = s.pvdone + 2;
+  s.mmadone = s.ofree + 1;
+  s.anc = s.mmadone + 1;
+  s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
+  s.tmem_base = reinterpret_cast<uint32_t*>(s.par + kMaxTreeNodes);
+  s.misc = reinterpret_cast<int*>(s.tmem_base + 4);
+  s.len = s.misc + 8;
+  s.base = s.len + C;
+  return s;
+}
+
+// ------------------------------------------------------------ MMA issuer
+
+struct PendingPV {
+  int stage, sb, tile, piece;
+  bool first;
+};
+
+__device__ __forceinline__ bool issue_pv(const AttnParams& p, const Smem& sm, uint32_t tmem, const PendingPV& pv) {
+  if (!mbar_wait(smem_addr(&sm.pfull[pv.sb]), (pv.tile >> 1) & 1, p.err)) return false;
+  if (pv.first && pv.piece > 0 && !mbar_wait(smem_addr(sm.ofree), (pv.piece - 1) & 1, p.err)) return false;
+  tc_fence_after();
+  constexpr uint32_t idesc = idesc_bf16(128, 128, true);
+  const uint32_t pbase = smem_addr(sm.pbuf + pv.sb * kPBufBytes);
+  const uint32_t vbase = smem_addr(sm.ring + static_cast<size_t>(pv.stage) * kStageBytes + kKVTileBytes);
+#pragma unroll
+  for (int kk = 0; kk < kTileKeys / 16; ++kk) {
+    const uint64_t a = smem_desc_sw128(pbase + kk * 32, 16, 1024);
+    // V tile is MN-major: 64-dim halves 8 KB apart (leading), 8-key groups 1 KB apart (stride).
+    const uint64_t b = smem_desc_sw128(vbase + kk * 2048, kHalfBytes, 1024);
+    tc_mma(tmem + kTmemO, a, b, idesc, (pv.first && kk == 0) ? 0u : 1u);
+  }
+  tc_commit(smem_addr(&sm.empty[pv.stage]));
+  tc_commit(smem_addr(&sm.pvdone[pv.sb]));
+  return true;
+}
+
+__device__ void run_mma(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem, Cursor cu) {
+  constexpr uint32_t idesc = idesc_bf16(128, 64, false);
+  int stage = 0, t = 0, piece = 0, qb = 0, cur_piece = 0;
+  uint32_t phase = 0;
+  PendingPV prev{0, 0, 0, 0, false};
+  bool have_prev = false, ok = true;
+  for (; cu.t < cu.t_end; cursor_next(cu, p, sm.len)) {
+    if (*pipe.abort) {
+      ok = false;
+      break;
+    }
+    const TileInfo ti = tile_info(cu, p);
+    if (ti.first) {
+      qb = piece & 1;
+      cur_piece = piece;
+      if (!mbar_wait(smem_addr(&sm.qfull[qb]), (piece >> 1) & 1, p.err)) {
+        ok = false;
+        break;
+      }
+      ++piece;
+    }
+    if (!mbar_wait(smem_addr(&pipe.full[stage]), phase, p.err)) {
+      ok = false;
+      break;
+    }
+    sm.misc[2] = t + 1;
+    tc_fence_after();
+    const int sb = t & 1;
+    const uint32_t qbase = smem_addr(sm.qbuf + qb * kQBufBytes);
+    const uint32_t kbase = smem_addr(sm.ring + static_cast<size_t>(stage) * kStageBytes);
+#pragma unroll
+    for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+      const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
+      const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * kHalfBytes + (ks & 3) * 32, 16, 1024);
+      tc_mma(tmem + sb * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
+    }
+    tc_commit(smem_addr(&sm.sfull[sb]));
+    if (ti.last) tc_commit(smem_addr(&sm.qempty[qb]));
+    if (have_prev && !issue_pv(p, sm, tmem, prev)) {
+      ok = false;
+      break;
+    }
+    prev = PendingPV{stage, sb, t, cur_piece, ti.first};
+    have_prev = true;
+    ++t;
+    if (++stage == kStages) {
+      stage = 0;
+      phase ^= 1u;
+    }
+  }
+  if (ok && have_prev) ok = issue_pv(p, sm, tmem, prev);
+  if (!ok) *pipe.abort = 1;
+  sm.misc[2] = t;      // tiles whose loads were waited for
+  sm.misc[4] = piece;  // q blocks whose loads were waited for
+  tc_commit(smem_addr(sm.mmadone));
+}
+
+// ------------------------------------------------------------ softmax + epilogue
+
+__device__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem, Cursor cu) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int quarter = warp & 3;                 // TMEM lanes this warp may access
+  const int r = quarter * 32 + lane;            // accumulator row of this thread
+  const int tid = threadIdx.x - 64;             // 0..127 among the softmax threads
+  const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+  const int HR = p.hkv * p.row_blocks;
+  // Kernel parameters used per element, read once (p refers to parameter space).
+  const float qscale = p.qscale;
+  const bool tree = p.tree != 0;
+  const int nq = p.Nq, n_nodes = p.N;
+  float m_run = -INFINITY, l_run = 0.f;
+  int t = 0, stage = 0, anc_seq = -1;
+  uint32_t phase = 0;
+  for (; cu.t < cu.t_end; cursor_next(cu, p, sm.len)) {
+    const TileInfo ti = tile_info(cu, p);
+    const int h = cu.hr / p.row_blocks, rb = cu.hr - h * p.row_blocks;
+    const int rows_blk = min(p.rows_per_unit, p.rows_total - rb * p.rows_per_unit);
+    const bool valid = r < rows_blk;
+    const bool warp_live = quarter * 32 < rows_blk;
+    const int rr = rb * p.rows_per_unit + r;
+    const int nl = valid ? rr / p.G : 0;
+    if (ti.first) {
+      m_run = -INFINITY;
+      l_run = 0.f;
+    }
+    if (ti.draft && p.tree) {
+      const int seq = cu.c / (p.C / p.B);
+      if (seq != anc_seq) {
+        build_ancestor_masks(p, seq, sm.anc, sm.par, tid, kSoftmaxThreads, kBarSoftmax);
+        anc_seq = seq;
+      }
+    }
+    const int sb = t & 1;
+    bool live = !*pipe.abort;
+    if (live && !mbar_wait(smem_addr(&sm.sfull[sb]), (t >> 1) & 1, p.err)) {
+      *pipe.abort = 1;
+      live = false;
+    }
+    live = __all_sync(0xffffffffu, live);
+    tc_fence_after();
+    uint32_t sv[64];
+    float pr[64];
+    if (live && warp_live) {
+      uint32_t lo[32], hi[32];
+      tmem_ld32(trow + sb * kTileKeys, lo);
+      tmem_ld32(trow + sb * kTileKeys + 32, hi);
+      tmem_wait_ld();
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        sv[j] = lo[j];
+        sv[32 + j] = hi[j];
+      }
+    }
+    if (live && warp_live) {
+      // Visible keys of this row in this tile as a 64-bit mask (bit j = key j of the tile).
+      uint64_t vis = 0;
+      if (valid) {
+        vis = ti.nkeys >= 64 ? ~0ull : ((1ull << ti.nkeys) - 1ull);
+        if (ti.draft) {
+          uint64_t dm;
+          if (tree) {
+            dm = sm.anc[min(nl, nq - 1)] >> ti.key0;  // tree drafts have N <= 64, so key0 == 0
+          } else {
+            const int last = n_nodes - nq + nl - ti.key0;  // chain: slots key0 .. node are visible
+            dm = last >= 63 ? ~0ull : (last < 0 ? 0ull : ((2ull << last) - 1ull));
+          }
+          vis &= dm;
+        }
+      }
+      float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+      for (int j = 0; j < 64; ++j) {
+        pr[j] = ((vis >> j) & 1ull) ? __uint_as_float(sv[j]) * qscale : -INFINITY;
+        mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
+      }
+      const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+      // Lazy rescale: move this row's reference max only when it grows by > 2^8.
+      const bool grow = valid && (m_run == -INFINITY ? mx != -INFINITY : mx > m_run + kRescaleThreshold);
+      const bool rescale_o = grow && m_run != -INFINITY;
+      if (__any_sync(0xffffffffu, rescale_o)) {
+        // O must hold P.V of the previous tile before it is scaled.
+        if (!mbar_wait(smem_addr(&sm.pvdone[(t - 1) & 1]), ((t - 1) >> 1) & 1, p.err)) *pipe.abort = 1;
+        tc_fence_after();
+        const float alpha = rescale_o ? ex2(m_run - mx) : 1.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[32];
+          tmem_ld32(trow + kTmemO + 32 * c, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha);
+          tmem_st32(trow + kTmemO + 32 * c, o);
+        }
+        tmem_wait_st();
+        l_run *= alpha;
+      }
+      if (grow) m_run = mx;
+      const float m_use = m_run == -INFINITY ? 0.f : m_run;
+      float ps4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int j = 0; j < 64; ++j) {
+        pr[j] = ex2(pr[j] - m_use);
+        ps4[j & 3] += pr[j];
+      }
+      l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
+    }
+    // The P buffer is free once P.V of tile t-2 has completed.
+    if (live && t >= 2 && !mbar_wait(smem_addr(&sm.pvdone[sb]), ((t - 2) >> 1) & 1, p.err)) *pipe.abort = 1;
+    if (live && valid) {
+      uint8_t* prow = sm.pbuf + sb * kPBufBytes + r * 128;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        uint4 w;
+        w.x = pack_bf16x2(pr[8 * c + 0], pr[8 * c + 1]);
+        w.y = pack_bf16x2(pr[8 * c + 2], pr[8 * c + 3]);
+        w.z = pack_bf16x2(pr[8 * c + 4], pr[8 * c + 5]);
+        w.w = pack_bf16x2(pr[8 * c + 6], pr[8 * c + 7]);
+        *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = w;
+      }
+    }
+    if (live && ti.nkeys < kTileKeys) {
+      // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.
+      if (!mbar_wait(smem_addr(&pipe.full[stage]), phase, p.err)) *pipe.abort = 1;
+      uint8_t* vptr = pipe.ring + static_cast<size_t>(stage) * kStageBytes + kKVTileBytes;
+      const int nz = (kTileKeys - ti.nkeys) * 16;
+      for (int i = tid; i < nz; i += kSoftmaxThreads) {
+        const int key = ti.nkeys + (i >> 4), ch = i & 15;
+        *reinterpret_cast<uint4*>(vptr + tile_off(key, ch)) = make_uint4(0, 0, 0, 0);
+      }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    mbar_arrive(smem_addr(&sm.pfull[sb]));
+    if (ti.last) {
+      bool ok = live && mbar_wait(smem_addr(&sm.pvdone[sb]), (t >> 1) & 1, p.err);
+      ok = __all_sync(0xffffffffu, ok);
+      tc_fence_after();
+      if (ok && warp_live) {
+        const bool whole = cu.lt == cu.ut - 1 && (cu.t - cu.t_begin) >= cu.lt;
+        const int slot = cu.c * HR + cu.hr + blockIdx.x;
+        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+        const float lse2 = l_run > 0.f ? m_run + __log2f(l_run) : -INFINITY;
+        size_t orow = 0;
+        if (valid && whole) {
+          const int g = rr - nl * p.G;
+          orow = (static_cast<size_t>(cu.c) * p.Nq + nl) * p.hq + h * p.G + g;
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[32];
+          tmem_ld32(trow + kTmemO + 32 * c, o);
+          tmem_wait_ld();
+          if (valid) {
+            if (whole) {
+              uint4* dst = reinterpret_cast<uint4*>(p.out + orow * kHeadDim + 32 * c);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                uint4 w;
+                w.x = pack_bf16x2(__uint_as_float(o[8 * k + 0]) * inv, __uint_as_float(o[8 * k + 1]) * inv);
+                w.y = pack_bf16x2(__uint_as_float(o[8 * k + 2]) * inv, __uint_as_float(o[8 * k + 3]) * inv);
+                w.z = pack_bf16x2(__uint_as_float(o[8 * k + 4]) * inv, __uint_as_float(o[8 * k + 5]) * inv);
+                w.w = pack_bf16x2(__uint_as_float(o[8 * k + 6]) * inv, __uint_as_float(o[8 * k + 7]) * inv);
+                dst[k] = w;
+              }
+            } else {
+              float4* dst = reinterpret_cast<float4*>(
+                  p.ws_o + (static_cast<size_t>(slot) * p.rows_per_unit + r) * kHeadDim + 32 * c);
+#pragma unroll
+              for (int k = 0; k < 8; ++k)
+                dst[k] = make_float4(__uint_as_float(o[4 * k]) * inv, __uint_as_float(o[4 * k + 1]) * inv,
+                                     __uint_as_float(o[4 * k + 2]) * inv, __uint_as_float(o[4 * k + 3]) * inv);
+            }
+          }
+        }
+        if (valid) {
+          if (whole) p.lse[orow] = lse2 * 0.69314718055994531f;
+          else p.ws_lse[static_cast<size_t>(slot) * p.rows_per_unit + r] = lse2;
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(smem_addr(sm.ofree));
+    }
+    ++t;
+    if (++stage == kStages) {
+      stage = 0;
+      phase ^= 1u;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_tc_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ TensorMaps maps, int nq_box) {
+  extern __shared__ uint8_t smem_raw[];
+  const Smem sm = carve(smem_raw, p.C);
+  const int warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(smem_addr(&sm.full[s]), 1);
+      mbar_init(smem_addr(&sm.empty[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_addr(&sm.qfull[b]), 1);
+      mbar_init(smem_addr(&sm.qempty[b]), 1);
+      mbar_init(smem_addr(&sm.sfull[b]), 1);
+      mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads);
+      mbar_init(smem_addr(&sm.pvdone[b]), 1);
+    }
+    mbar_init(smem_addr(sm.ofree), kSoftmaxThreads);
+    mbar_init(smem_addr(sm.mmadone), 1);
+    for (int i = 0; i < 8; ++i) sm.misc[i] = 0;
+    fence_mbar_init();
+    prefetch_tensormap(&maps.tk);
+    prefetch_tensormap(&maps.tv);
+    prefetch_tensormap(&maps.dk);
+    prefetch_tensormap(&maps.dv);
+    prefetch_tensormap(&maps.q);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_addr(sm.tmem_base), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  build_plan(p, sm.len, sm.base);  // block-wide barriers inside
+  tc_fence_after();
+  const uint32_t tmem = *sm.tmem_base;
+  const Cursor cu = cursor_begin(p, sm.len, sm.base);
+  Pipe pipe{sm.ring, sm.full, sm.empty, kStages, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
+  QPipe qp{sm.qbuf, sm.qfull, sm.qempty, p.G * nq_box, nq_box, &sm.misc[3]};
+  if (warp == 0) {
+    run_producer(p, maps, pipe, sm.len, cu, &qp);
+  } else if (warp == 1) {
+    if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
+      run_mma(p, sm, pipe, tmem, cu);
+      // Every MMA must have completed before TMEM is released.
+      mbar_wait(smem_addr(sm.mmadone), 0, p.err);
+    }
+    __syncwarp();
+  } else {
+    run_softmax(p, sm, pipe, tmem, cu);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (threadIdx.x == 0 && *pipe.abort) {
+    // A wait timed out: let every TMA load still in flight land before the CTA exits.
+    drain_after_abort(p, pipe, sm.misc[2]);
+    for (int k = sm.misc[4]; k < sm.misc[3]; ++k)
+      if (!mbar_wait(smem_addr(&sm.qfull[k & 1]), (k >> 1) & 1, p.err)) break;
+  }
+  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+}  // namespace
+
+cudaError_t attn_tc_occupancy(int C, int* ctas_per_sm) {
+  const size_t smem = smem_bytes(C);
+  cudaError_t e =
+      cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, attn_tc_kernel, kThreads, smem);
+}
+
+cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, cudaStream_t stream) {
+  const size_t smem = smem_bytes(p.C);
+  cudaError_t e =
+      cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  attn_tc_kernel<<<p.num_ctas, kThreads, smem, stream>>>(p, maps, nq_box);
+  return cudaGetLastError();
+}
+
+}  // namespace kvshot

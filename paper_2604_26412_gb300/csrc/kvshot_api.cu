@@ -16,6 +16,7 @@ namespace kvshot {
 // Defined in the kernel translation units.
 cudaError_t attn_cc_occupancy(int C, int* ctas_per_sm);
 cudaError_t attn_mma_occupancy(int m_tiles, int C, int* ctas_per_sm);
+cudaError_t attn_tc_occupancy(int C, int* ctas_per_sm);
 
 namespace {
 
@@ -52,9 +53,29 @@ bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+enum class Kernel { kCudaCore, kMma, kTensorMemory };
+
+// 4-D view {128 dims, hq, Nq, C} of q [C, Nq, hq, 128]; a box is one 64-dim
+// half of the G heads of one KV group for nq_box draft nodes (rows node-major).
+bool encode_q(CUtensorMap* map, const void* q, int C, int Nq, int hq, int G, int nq_box) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[4] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(hq),
+                              static_cast<cuuint64_t>(Nq), static_cast<cuuint64_t>(C)};
+  const cuuint64_t row = static_cast<cuuint64_t>(kHeadDim) * 2;
+  const cuuint64_t strides[3] = {row, row * hq, row * hq * Nq};
+  const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(nq_box), 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(q), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct Plan {
+  Kernel kernel;
   bool mma;
   int m_tiles;        // mma path
+  int nq_box;         // tensor-memory path: draft nodes per 128-row block
   int rows_per_unit;
   int row_blocks;
   int units;
@@ -85,9 +106,12 @@ kvshot_status check_common(const kvshot_attn_desc* d) {
   if (d->n_nodes < 0 || d->n_query < 0 || d->n_query > d->n_nodes || d->n_nodes > d->n_max) return KVSHOT_ERR_SHAPE;
   if (d->max_seq_len < 0) return KVSHOT_ERR_SHAPE;
   if (!std::isfinite(d->scale)) return KVSHOT_ERR_SHAPE;
-  const uint32_t known = KVSHOT_TREE | KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA;
+  const uint32_t known = KVSHOT_TREE | KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC;
   if ((d->flags & ~known) != 0) return KVSHOT_ERR_SHAPE;
-  if ((d->flags & KVSHOT_FORCE_CC) && (d->flags & KVSHOT_FORCE_MMA)) return KVSHOT_ERR_SHAPE;
+  const uint32_t force = d->flags & (KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC);
+  if (force & (force - 1)) return KVSHOT_ERR_SHAPE;  // at most one kernel may be forced
+  const int G = d->hq / d->hkv;
+  if ((d->flags & KVSHOT_FORCE_TC) && (G > 128 || 128 % G != 0)) return KVSHOT_ERR_UNSUPPORTED;
   if ((d->flags & KVSHOT_TREE) && d->n_nodes > kMaxTreeNodes) return KVSHOT_ERR_UNSUPPORTED;
   if (d->num_ctas < 0) return KVSHOT_ERR_SHAPE;
   if (static_cast<int64_t>(d->num_caches) * d->hkv * d->n_max >= INT_MAX) return KVSHOT_ERR_UNSUPPORTED;
@@ -114,19 +138,23 @@ kvshot_status check_attn_desc(const kvshot_attn_desc* d, bool paged) {
 kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   const int G = d->hq / d->hkv;
   const int rows = G * d->n_query;
-  const bool force_cc = d->flags & KVSHOT_FORCE_CC, force_mma = d->flags & KVSHOT_FORCE_MMA;
+  const bool force_cc = d->flags & KVSHOT_FORCE_CC, force_tc = d->flags & KVSHOT_FORCE_TC;
   // Measured on GB300 (ncu + bench): at 4 stacked rows the CUDA-core kernel is
   // issue/latency bound (IPC ~1, ~100 warp instructions per key) while the
   // m16n8k16 kernel, with the stack zero-padded to 16 rows, streams K/V at
   // 73-97% of HBM bandwidth; so the tensor-core kernel is the default for every
   // stack size and the CUDA-core kernel is kept behind KVSHOT_FORCE_CC.
-  (void)force_mma;
-  pl->mma = !force_cc;
-  if (pl->mma) {
+  pl->kernel = force_cc ? Kernel::kCudaCore : force_tc ? Kernel::kTensorMemory : Kernel::kMma;
+  pl->mma = pl->kernel == Kernel::kMma;
+  pl->m_tiles = 0;
+  pl->nq_box = 0;
+  if (pl->kernel == Kernel::kMma) {
     pl->m_tiles = std::min(kMmaMaxTiles, std::max(1, (rows + 15) / 16));
     pl->rows_per_unit = 16 * pl->m_tiles;
+  } else if (pl->kernel == Kernel::kTensorMemory) {
+    pl->nq_box = std::max(1, std::min(d->n_query, 128 / G));
+    pl->rows_per_unit = G * pl->nq_box;
   } else {
-    pl->m_tiles = 0;
     pl->rows_per_unit = kCcRows;
   }
   pl->row_blocks = std::max(1, (rows + pl->rows_per_unit - 1) / pl->rows_per_unit);
@@ -143,8 +171,9 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   int grid = d->num_ctas;
   if (grid == 0) {
     int per_sm = 0;
-    const cudaError_t e = pl->mma ? attn_mma_occupancy(pl->m_tiles, d->num_caches, &per_sm)
-                                  : attn_cc_occupancy(d->num_caches, &per_sm);
+    const cudaError_t e = pl->kernel == Kernel::kMma ? attn_mma_occupancy(pl->m_tiles, d->num_caches, &per_sm)
+                          : pl->kernel == Kernel::kTensorMemory ? attn_tc_occupancy(d->num_caches, &per_sm)
+                                                                 : attn_cc_occupancy(d->num_caches, &per_sm);
     const int sms = sm_count();
     if (e != cudaSuccess || per_sm < 1 || sms < 1) return KVSHOT_ERR_CUDA;
     grid = sms * per_sm;
@@ -217,6 +246,11 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   if (!encode_rows(&maps.tk, target_k, trows, tbox) || !encode_rows(&maps.tv, target_v, trows, tbox) ||
       !encode_rows(&maps.dk, draft_k, drows, kDraftBoxRows) || !encode_rows(&maps.dv, draft_v, drows, kDraftBoxRows))
     return KVSHOT_ERR_CUDA;
+  if (pl.kernel == Kernel::kTensorMemory) {
+    if (!encode_q(&maps.q, q, d->num_caches, d->n_query, d->hq, d->hq / d->hkv, pl.nq_box)) return KVSHOT_ERR_CUDA;
+  } else {
+    maps.q = maps.tk;  // unused by the other kernels
+  }
 
   AttnParams p;
   p.q = static_cast<const __nv_bfloat16*>(q);
@@ -255,7 +289,9 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   p.num_ctas = pl.num_ctas;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  cudaError_t e = pl.mma ? launch_attn_mma(p, maps, pl.m_tiles, s) : launch_attn_cc(p, maps, s);
+  cudaError_t e = pl.kernel == Kernel::kMma            ? launch_attn_mma(p, maps, pl.m_tiles, s)
+                  : pl.kernel == Kernel::kTensorMemory ? launch_attn_tc(p, maps, pl.nq_box, s)
+                                                       : launch_attn_cc(p, maps, s);
   if (e != cudaSuccess) return KVSHOT_ERR_CUDA;
   e = launch_merge(p, s);
   return e == cudaSuccess ? KVSHOT_OK : KVSHOT_ERR_CUDA;

@@ -96,6 +96,16 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// 4-D tiled TMA load (default L2 policy).
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int x, int y, int z, int w,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(bar)
+      : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -338,15 +348,29 @@ struct Pipe {
   int* issued;         // tiles issued by the producer
 };
 
+// Double-buffered q staging (tensor-memory kernel only): piece k's query
+// block goes to buffer k % 2 (two 64-dim halves of 128 rows, 128B-swizzled).
+struct QPipe {
+  uint8_t* buf;        // 2 x kQBufBytes, 1024-aligned
+  uint64_t* full;      // [2] TMA -> MMA issuer
+  uint64_t* empty;     // [2] MMA completion -> TMA
+  int rows;            // rows loaded per box (G x nodes per box)
+  int nq_box;          // draft nodes per box
+  int* issued;         // q blocks issued
+};
+constexpr int kQRows = 128;
+constexpr int kQBufBytes = 2 * kQRows * 128;
+
 // The producer warp: walks this CTA's tiles and issues their TMA loads into the
 // stage ring, one tile ahead on the page-table reads.  Lane 0 issues.
 __device__ void run_producer(const AttnParams& p, const TensorMaps& maps, const Pipe& pipe, const int* s_len,
-                             Cursor cu) {
+                             Cursor cu, const QPipe* qp = nullptr) {
   const int lane = threadIdx.x & 31;
   const uint64_t policy = l2_policy_evict_first();
   int stage = 0;
   uint32_t phase = 0;
   int issued = 0;
+  int piece = 0;
   int pid_cur = tile_page_ids(p, cu, lane);
   while (cu.t < cu.t_end) {
     Cursor nx = cu;
@@ -365,7 +389,26 @@ __device__ void run_producer(const AttnParams& p, const TensorMaps& maps, const 
     for (int i = 0; i < kTileKeys / 8; ++i) pids[i] = __shfl_sync(0xffffffffu, pid_cur, i);
 
     int ok = 1;
-    if (lane == 0) {
+    if (qp != nullptr && (cu.t == cu.t_begin || cu.lt == 0)) {
+      // First tile of a piece: stage the unit's query block (all its G x Nq rows).
+      if (lane == 0) {
+        const int qb = piece & 1;
+        const uint32_t qbar = smem_addr(&qp->full[qb]);
+        ok = mbar_wait(smem_addr(&qp->empty[qb]), ((piece >> 1) & 1) ^ 1u, p.err) ? 1 : 0;
+        if (ok && !*pipe.abort) {
+          const int rb = cu.hr - h * p.row_blocks;
+          const uint32_t dst = smem_addr(qp->buf + qb * kQBufBytes);
+          mbar_arrive_expect_tx(qbar, 2 * qp->rows * 128);
+          tma_load_4d(dst, &maps.q, 0, h * p.G, rb * qp->nq_box, cu.c, qbar);
+          tma_load_4d(dst + kQRows * 128, &maps.q, 64, h * p.G, rb * qp->nq_box, cu.c, qbar);
+          *qp->issued = piece + 1;
+        } else {
+          ok = 0;
+        }
+      }
+      ++piece;
+    }
+    if (lane == 0 && ok) {
       ok = mbar_wait(smem_addr(&pipe.empty[stage]), phase ^ 1u, p.err) ? 1 : 0;
       if (!ok || *pipe.abort) ok = 0;
     }

@@ -72,11 +72,13 @@ struct AppendParams {
 
 struct TensorMaps {
   CUtensorMap tk, tv, dk, dv;
+  CUtensorMap q;  // [C, Nq, hq, 128] as 4-D {128, hq, Nq, C}; used by the tensor-memory kernel
 };
 
 // Kernel launchers (one per translation unit).  Return cudaSuccess or the launch error.
 cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, cudaStream_t stream);
 cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, cudaStream_t stream);
+cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, cudaStream_t stream);
 cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream);
 cudaError_t launch_append(const AppendParams& a, cudaStream_t stream);
 

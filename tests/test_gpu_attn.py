@@ -76,16 +76,18 @@ def test_attn_matches_oracle(case):
     spec, inp, dk, dv, q, N, Nq = _case(lens, levels, tree, paged, P, hq, hkv, nq, seed=len(lens) + N_SEED(case))
     hc = gh.HostCache(inp)
     ref_out, ref_lse = gh.oracle_attn(hc, q, dk, dv, N, Nq)
-    for num_ctas in (0, 1, 7):
-        out, lse = _run(spec, inp, dk, dv, q, N, Nq, num_ctas=num_ctas)
-        gh.compare(out, lse, ref_out, ref_lse, f"{case} ctas={num_ctas}")
+    kernels = [0, kvshot.KVSHOT_FORCE_TC] if 128 % (hq // hkv) == 0 else [0]
+    for flags in kernels:
+        for num_ctas in (0, 1, 7):
+            out, lse = _run(spec, inp, dk, dv, q, N, Nq, flags=flags, num_ctas=num_ctas)
+            gh.compare(out, lse, ref_out, ref_lse, f"{case} flags={flags} ctas={num_ctas}")
 
 
 def N_SEED(case):
     return sum(case[1]) * 7 + (3 if case[2] else 0)
 
 
-@pytest.mark.parametrize("flags", [kvshot.KVSHOT_FORCE_CC, kvshot.KVSHOT_FORCE_MMA])
+@pytest.mark.parametrize("flags", [kvshot.KVSHOT_FORCE_CC, kvshot.KVSHOT_FORCE_MMA, kvshot.KVSHOT_FORCE_TC])
 @pytest.mark.parametrize("nq", [1, 3, 8])
 def test_forced_kernels_agree_with_oracle(flags, nq):
     spec, inp, dk, dv, q, N, Nq = _case((300, 77), (2, 3, 3), True, True, 16, 32, 8, nq, seed=11)
@@ -112,9 +114,10 @@ def test_deterministic_across_runs():
     assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
 
 
+@pytest.mark.parametrize("flags", [0, kvshot.KVSHOT_FORCE_TC])
 @pytest.mark.parametrize("paged", [False, True])
 @pytest.mark.parametrize("tree", [False, True])
-def test_mask_probe_is_exact(paged, tree):
+def test_mask_probe_is_exact(paged, tree, flags):
     """q = 0 and one-hot V: every visible draft slot contributes exactly 1/n_vis to its own bucket."""
     lens = (37, 64, 129, 0) if paged else (37, 64, 129, 5)
     levels = (3, 5, 8, 8, 4) if tree else (1,) * 12
@@ -133,7 +136,7 @@ def test_mask_probe_is_exact(paged, tree):
     dv[:, :, :N].zero_()
     for m in range(N):
         dv[:, :, m, 64 + m] = 1.0
-    out, lse = _run(spec, inp, dk, dv, q, N, Nq)
+    out, lse = _run(spec, inp, dk, dv, q, N, Nq, flags=flags)
     parents = inp.tree_parent.cpu().numpy()
     o = out.float().cpu().numpy()
     l = lse.cpu().numpy()
