@@ -79,7 +79,7 @@ __device__ __forceinline__ void unpack16(const uint4& a, const uint4& b, float (
 
 // Final or partial write of one unit piece: combine the 4 consumer warps'
 // (m, l, o) states through shared memory.
-__device__ void finalize(const AttnParams& p, const Smem& sm, int c, int h, int rb, int slot, bool whole,
+__device__ __forceinline__ void finalize(const AttnParams& p, const Smem& sm, int c, int h, int rb, int slot, bool whole,
                          float (&o)[kCcRows][16], const float (&m_run)[kCcRows], float (&l_run)[kCcRows]) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int grp = lane >> 3, s8 = lane & 7;
@@ -155,7 +155,7 @@ __device__ void finalize(const AttnParams& p, const Smem& sm, int c, int h, int 
   named_barrier_sync(kBarConsumers, kWarps * 32);
 }
 
-__device__ void run_consumer(const AttnParams& p, const Smem& sm, const Pipe& pipe, Cursor cu) {
+__device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm, const Pipe& pipe, Cursor cu) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int grp = lane >> 3, s8 = lane & 7;
   float qf[kCcRows][16];

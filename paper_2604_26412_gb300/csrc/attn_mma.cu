@@ -80,7 +80,7 @@ __device__ Smem carve(uint8_t* raw, int C) {
 // final bf16 output + lse if the piece is the whole unit, else the
 // normalised fp32 partial + log2-domain lse into workspace slot `slot`.
 template <class CF>
-__device__ void finalize(const AttnParams& p, const Smem& sm, int c, int h, int rb, int slot, bool whole,
+__device__ __forceinline__ void finalize(const AttnParams& p, const Smem& sm, int c, int h, int rb, int slot, bool whole,
                          float (&o)[16][4], const float (&m_run)[2], float (&l_run)[2]) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int mt = warp % CF::kMT, ks = warp / CF::kMT;
@@ -180,7 +180,7 @@ __device__ void finalize(const AttnParams& p, const Smem& sm, int c, int h, int 
 }
 
 template <class CF>
-__device__ void run_consumer(const AttnParams& p, const Smem& sm, const Pipe& pipe, Cursor cu) {
+__device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm, const Pipe& pipe, Cursor cu) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int mt = warp % CF::kMT, ks = warp / CF::kMT;
   const int g = lane >> 2, q4 = lane & 3;

@@ -7,12 +7,18 @@
 //   S = Q K^T      tcgen05.mma M=128 N=64  K=128 (8 x K16), A = Q (smem), B = K tile (smem), D = S (TMEM)
 //   P = softmax(S) one thread per row: TMEM -> registers -> bf16 P (smem, 128B-swizzled)
 //   O += P V       tcgen05.mma M=128 N=128 K=64 (4 x K16), A = P (smem), B = V tile (smem, MN-major), D = O (TMEM)
-// Warp roles: warp 0 issues TMA (K/V tiles, one q block per piece), warp 1
-// owns TMEM and one of its threads issues every MMA, warps 2..5 run the
-// softmax and the epilogue (thread = TMEM lane = row).  S is double-buffered
-// in TMEM so QK^T of tile t+1 overlaps the softmax of tile t; O is rescaled in
-// TMEM only when a row's running max grows by more than 2^8 (lazy rescale).
-// Rows of the 128-row MMA beyond the unit's stack carry no output.
+// Warp roles: warps 0..7 are two softmax warpgroups, warp 10 issues TMA
+// (K/V tiles, one q block per piece), warp 11 owns TMEM and one of its
+// threads issues every MMA (warps 8, 9 idle).  A warp issues from SM
+// sub-partition warp % 4; the TMA and MMA warps sit on sub-partitions 2 and 3,
+// away from the rows 0..31 softmax warps that small GQA stacks keep busiest.  Warpgroup w takes key columns [32w, 32w+32) of every
+// tile with its own running max/sum and its own O accumulator O_w in TMEM
+// (thread = TMEM lane = row); the two are merged by log-sum-exp at the end of
+// each piece.  S has four TMEM buffers; the MMA thread issues QK^T as soon as
+// a K tile and an S buffer are free and P.V as soon as P is written, so QK^T
+// runs ahead of the softmax and the in-order MMA latency hides behind it.  O_w is rescaled in TMEM only
+// when a row's running max grows by more than 2^8 (lazy rescale).  Rows of
+// the 128-row MMA beyond the unit's stack carry no output.
 #include "kvshot_attn_common.cuh"
 
 namespace kvshot {
@@ -20,13 +26,17 @@ namespace {
 
 using namespace dev;
 
-constexpr int kStages = 3;
-constexpr int kThreads = 6 * 32;
-constexpr int kSoftmaxThreads = 128;
+constexpr int kStages = 4;                 // K/V ring
+constexpr int kNS = 4;                     // S buffers in TMEM: QK^T may run up to 4 tiles ahead of P.V
+constexpr int kNP = 3;                     // P buffers in shared memory
+constexpr int kThreads = 12 * 32;
+constexpr int kProducerWarp = 10;
+constexpr int kMmaWarp = 11;
+constexpr int kSoftmaxThreads = 256;       // two warpgroups
 constexpr int kBarSoftmax = 1;             // named barrier among the softmax warps
 constexpr int kPBufBytes = kQRows * 128;   // 128 rows x 64 keys bf16
-constexpr uint32_t kTmemCols = 256;        // S0 [0,64) S1 [64,128) O [128,256)
-constexpr uint32_t kTmemO = 128;
+constexpr uint32_t kTmemCols = 512;        // S0..S3 [0,256), O0 [256,384), O1 [384,512)
+constexpr uint32_t kTmemO = kNS * kTileKeys;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max grows by > 256x
 
 // ------------------------------------------------------------ tcgen05 wrappers
@@ -111,19 +121,20 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major)
 
 struct Smem {
   uint8_t* ring;       // kStages x (K tile | V tile)
-  uint8_t* qbuf;       // 2 x kQBufBytes
-  uint8_t* pbuf;       // 2 x kPBufBytes
+  uint8_t* qbuf;       // one q block
+  uint8_t* pbuf;       // kNP x kPBufBytes
   uint64_t* full;      // [kStages]
   uint64_t* empty;     // [kStages]  (MMA completion)
-  uint64_t* qfull;     // [2]
-  uint64_t* qempty;    // [2]
-  uint64_t* sfull;     // [2]  S buffer written (MMA completion)
-  uint64_t* pfull;     // [2]  P buffer written (128 softmax threads)
-  uint64_t* pvdone;    // [2]  P.V of the tile using that buffer completed
+  uint64_t* qfull;     // [1]
+  uint64_t* qempty;    // [1]
+  uint64_t* sfull;     // [kNS]  S buffer written (MMA completion)
+  uint64_t* pfull;     // [kNP]  P buffer written and S consumed (256 softmax threads)
+  uint64_t* pvdone;    // [kNP]  P.V of the tile using that buffer completed
   uint64_t* ofree;     // [1]  epilogue finished reading O
   uint64_t* mmadone;   // [1]  every MMA completed
   uint64_t* anc;       // [64]
   int* par;            // [64]
+  float* comb;         // [128][2] second warpgroup's (max, sum) per row at a piece end
   uint32_t* tmem_base;
   int* misc;           // [0] abort, [1] tiles issued, [2] tiles consumed, [3] q blocks issued, [4] q consumed
   int* len;
@@ -131,9 +142,10 @@ struct Smem {
 };
 
 __host__ __device__ inline size_t smem_bytes(int C) {
-  size_t off = static_cast<size_t>(kStages) * kStageBytes + 2 * kQBufBytes + 2 * kPBufBytes;
-  off += sizeof(uint64_t) * (2 * kStages + 2 * 5 + 2);
+  size_t off = static_cast<size_t>(kStages) * kStageBytes + kQBufBytes + kNP * kPBufBytes;
+  off += sizeof(uint64_t) * (2 * kStages + 2 + kNS + 2 * kNP + 2);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
+  off += sizeof(float) * 2 * kQRows;
   off += sizeof(uint32_t) * 4 + sizeof(int) * 8;
   off += sizeof(int) * (2 * C + 1);
   return off + 1024;
@@ -145,22 +157,23 @@ __device__ Smem carve(uint8_t* raw, int C) {
   s.ring = p;
   p += kStages * kStageBytes;
   s.qbuf = p;
-  p += 2 * kQBufBytes;
+  p += kQBufBytes;
   s.pbuf = p;
-  p += 2 * kPBufBytes;
+  p += kNP * kPBufBytes;
   uint64_t* b = reinterpret_cast<uint64_t*>(p);
   s.full = b;
   s.empty = s.full + kStages;
   s.qfull = s.empty + kStages;
-  s.qempty = s.qfull + 2;
-  s.sfull = s.qempty + 2;
-  s.pfull = s.sfull + 2;
-  s.pvdone = s.pfull + 2;
-  s.ofree = s.pvdone + 2;
+  s.qempty = s.qfull + 1;
+  s.sfull = s.qempty + 1;
+  s.pfull = s.sfull + kNS;
+  s.pvdone = s.pfull + kNP;
+  s.ofree = s.pvdone + kNP;
   s.mmadone = s.ofree + 1;
   s.anc = s.mmadone + 1;
   s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
-  s.tmem_base = reinterpret_cast<uint32_t*>(s.par + kMaxTreeNodes);
+  s.comb = reinterpret_cast<float*>(s.par + kMaxTreeNodes);
+  s.tmem_base = reinterpret_cast<uint32_t*>(s.comb + 2 * kQRows);
   s.misc = reinterpret_cast<int*>(s.tmem_base + 4);
   s.len = s.misc + 8;
   s.base = s.len + C;
@@ -170,96 +183,118 @@ __device__ Smem carve(uint8_t* raw, int C) {
 // ------------------------------------------------------------ MMA issuer
 
 struct PendingPV {
-  int stage, sb, tile, piece;
+  int stage, tile, piece;
   bool first;
 };
 
-__device__ __forceinline__ bool issue_pv(const AttnParams& p, const Smem& sm, uint32_t tmem, const PendingPV& pv) {
-  if (!mbar_wait(smem_addr(&sm.pfull[pv.sb]), (pv.tile >> 1) & 1, p.err)) return false;
-  if (pv.first && pv.piece > 0 && !mbar_wait(smem_addr(sm.ofree), (pv.piece - 1) & 1, p.err)) return false;
-  tc_fence_after();
-  constexpr uint32_t idesc = idesc_bf16(128, 128, true);
-  const uint32_t pbase = smem_addr(sm.pbuf + pv.sb * kPBufBytes);
-  const uint32_t vbase = smem_addr(sm.ring + static_cast<size_t>(pv.stage) * kStageBytes + kKVTileBytes);
-#pragma unroll
-  for (int kk = 0; kk < kTileKeys / 16; ++kk) {
-    const uint64_t a = smem_desc_sw128(pbase + kk * 32, 16, 1024);
-    // V tile is MN-major: 64-dim halves 8 KB apart (leading), 8-key groups 1 KB apart (stride).
-    const uint64_t b = smem_desc_sw128(vbase + kk * 2048, kHalfBytes, 1024);
-    tc_mma(tmem + kTmemO, a, b, idesc, (pv.first && kk == 0) ? 0u : 1u);
-  }
-  tc_commit(smem_addr(&sm.empty[pv.stage]));
-  tc_commit(smem_addr(&sm.pvdone[pv.sb]));
-  return true;
+// O_w += P[:, 32w..32w+32) V[32w..32w+32, :] for both warpgroups w.
+__device__ __forceinline__ bool pv_ready(const Smem& sm, const PendingPV& pv) {
+  if (!mbar_test_wait(smem_addr(&sm.pfull[pv.tile % kNP]), (pv.tile / kNP) & 1)) return false;
+  return !(pv.first && pv.piece > 0) || mbar_test_wait(smem_addr(sm.ofree), (pv.piece - 1) & 1);
 }
 
-__device__ void run_mma(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem, Cursor cu) {
-  constexpr uint32_t idesc = idesc_bf16(128, 64, false);
-  int stage = 0, t = 0, piece = 0, qb = 0, cur_piece = 0;
-  uint32_t phase = 0;
-  PendingPV prev{0, 0, 0, 0, false};
-  bool have_prev = false, ok = true;
-  for (; cu.t < cu.t_end; cursor_next(cu, p, sm.len)) {
-    if (*pipe.abort) {
-      ok = false;
-      break;
-    }
-    const TileInfo ti = tile_info(cu, p);
-    if (ti.first) {
-      qb = piece & 1;
-      cur_piece = piece;
-      if (!mbar_wait(smem_addr(&sm.qfull[qb]), (piece >> 1) & 1, p.err)) {
-        ok = false;
-        break;
-      }
-      ++piece;
-    }
-    if (!mbar_wait(smem_addr(&pipe.full[stage]), phase, p.err)) {
-      ok = false;
-      break;
-    }
-    sm.misc[2] = t + 1;
-    tc_fence_after();
-    const int sb = t & 1;
-    const uint32_t qbase = smem_addr(sm.qbuf + qb * kQBufBytes);
-    const uint32_t kbase = smem_addr(sm.ring + static_cast<size_t>(stage) * kStageBytes);
+__device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, const PendingPV& pv) {
+  const int b = pv.tile % kNP;
+  tc_fence_after();
+  constexpr uint32_t idesc = idesc_bf16(128, 128, true);
+  const uint32_t pbase = smem_addr(sm.pbuf + b * kPBufBytes);
+  const uint32_t vbase = smem_addr(sm.ring + static_cast<size_t>(pv.stage) * kStageBytes + kKVTileBytes);
 #pragma unroll
-    for (int ks = 0; ks < kHeadDim / 16; ++ks) {
-      const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
-      const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * kHalfBytes + (ks & 3) * 32, 16, 1024);
-      tc_mma(tmem + sb * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
+  for (int w = 0; w < 2; ++w)
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      const int k16 = 2 * w + kk;  // 16-key step of the tile
+      const uint64_t a = smem_desc_sw128(pbase + k16 * 32, 16, 1024);
+      // V tile is MN-major: 64-dim halves 8 KB apart (leading), 8-key groups 1 KB apart (stride).
+      const uint64_t bd = smem_desc_sw128(vbase + k16 * 2048, kHalfBytes, 1024);
+      tc_mma(tmem + kTmemO + 128 * w, a, bd, idesc, (pv.first && kk == 0) ? 0u : 1u);
     }
-    tc_commit(smem_addr(&sm.sfull[sb]));
-    if (ti.last) tc_commit(smem_addr(&sm.qempty[qb]));
-    if (have_prev && !issue_pv(p, sm, tmem, prev)) {
+  tc_commit(smem_addr(&sm.empty[pv.stage]));
+  tc_commit(smem_addr(&sm.pvdone[b]));
+}
+
+// Event-driven issue: each pass issues QK^T of the next tile if its K tile has
+// landed and an S buffer is free, and P.V of the oldest pending tile if its P
+// is written.  Nothing blocks, so QK^T runs ahead of the softmax.
+__device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
+                                        Cursor cu) {
+  constexpr uint32_t idesc = idesc_bf16(128, 64, false);
+  int stage = 0, next_qk = 0, next_pv = 0, piece = 0, cur_piece = 0;
+  uint32_t phase = 0;
+  bool q_ready = false;  // the q block of the tile at the cursor is resident
+  PendingPV pend[kNS];
+  uint64_t idle_since = 0;
+  bool ok = true;
+  while (ok) {
+    bool progressed = false;
+    if (cu.t < cu.t_end && next_qk - next_pv < kNS) {
+      const TileInfo ti = tile_info(cu, p);
+      if (ti.first && !q_ready) q_ready = mbar_test_wait(smem_addr(sm.qfull), piece & 1);
+      if ((!ti.first || q_ready) && mbar_test_wait(smem_addr(&pipe.full[stage]), phase)) {
+        if (ti.first) {
+          cur_piece = piece++;
+          sm.misc[4] = piece;
+          q_ready = false;
+        }
+        sm.misc[2] = next_qk + 1;
+        tc_fence_after();
+        const uint32_t qbase = smem_addr(sm.qbuf);
+        const uint32_t kbase = smem_addr(sm.ring + static_cast<size_t>(stage) * kStageBytes);
+#pragma unroll
+        for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+          const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
+          const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * kHalfBytes + (ks & 3) * 32, 16, 1024);
+          tc_mma(tmem + (next_qk % kNS) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
+        }
+        tc_commit(smem_addr(&sm.sfull[next_qk % kNS]));
+        if (ti.last) tc_commit(smem_addr(sm.qempty));
+        pend[next_qk % kNS] = PendingPV{stage, next_qk, cur_piece, ti.first};
+        ++next_qk;
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+        cursor_next(cu, p, sm.len);
+        progressed = true;
+      }
+    }
+    if (next_pv < next_qk && pv_ready(sm, pend[next_pv % kNS])) {
+      issue_pv(sm, tmem, pend[next_pv % kNS]);
+      ++next_pv;
+      progressed = true;
+    }
+    if (cu.t >= cu.t_end && next_pv == next_qk) break;
+    if (progressed) {
+      idle_since = 0;
+    } else if (*pipe.abort) {
       ok = false;
-      break;
-    }
-    prev = PendingPV{stage, sb, t, cur_piece, ti.first};
-    have_prev = true;
-    ++t;
-    if (++stage == kStages) {
-      stage = 0;
-      phase ^= 1u;
+    } else {
+      const uint64_t now = global_timer_ns();
+      if (idle_since == 0) {
+        idle_since = now;
+      } else if (now - idle_since > kWaitLimitNs) {
+        set_error(p.err, KVSHOT_ERR_TIMEOUT);
+        ok = false;
+      }
     }
   }
-  if (ok && have_prev) ok = issue_pv(p, sm, tmem, prev);
   if (!ok) *pipe.abort = 1;
-  sm.misc[2] = t;      // tiles whose loads were waited for
-  sm.misc[4] = piece;  // q blocks whose loads were waited for
   tc_commit(smem_addr(sm.mmadone));
 }
 
 // ------------------------------------------------------------ softmax + epilogue
 
-__device__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem, Cursor cu) {
+__device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
+                                            Cursor cu) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int quarter = warp & 3;                 // TMEM lanes this warp may access
+  const int wg = warp >> 2;                     // warpgroup: key columns [32 wg, 32 wg + 32)
   const int r = quarter * 32 + lane;            // accumulator row of this thread
-  const int tid = threadIdx.x - 64;             // 0..127 among the softmax threads
+  const int tid = threadIdx.x;                  // 0..255 among the softmax threads
   const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+  const uint32_t my_o = trow + kTmemO + 128 * wg;
   const int HR = p.hkv * p.row_blocks;
-  // Kernel parameters used per element, read once (p refers to parameter space).
+  // Kernel parameters used per element, read once.
   const float qscale = p.qscale;
   const bool tree = p.tree != 0;
   const int nq = p.Nq, n_nodes = p.N;
@@ -278,39 +313,30 @@ __device__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pip
       m_run = -INFINITY;
       l_run = 0.f;
     }
-    if (ti.draft && p.tree) {
+    if (ti.draft && tree) {
       const int seq = cu.c / (p.C / p.B);
       if (seq != anc_seq) {
         build_ancestor_masks(p, seq, sm.anc, sm.par, tid, kSoftmaxThreads, kBarSoftmax);
         anc_seq = seq;
       }
     }
-    const int sb = t & 1;
+    const int sbuf = t % kNS, b = t % kNP;
     bool live = !*pipe.abort;
-    if (live && !mbar_wait(smem_addr(&sm.sfull[sb]), (t >> 1) & 1, p.err)) {
+    if (live && !mbar_wait(smem_addr(&sm.sfull[sbuf]), (t / kNS) & 1, p.err)) {
       *pipe.abort = 1;
       live = false;
     }
     live = __all_sync(0xffffffffu, live);
     tc_fence_after();
-    uint32_t sv[64];
-    float pr[64];
+    float pr[32];
     if (live && warp_live) {
-      uint32_t lo[32], hi[32];
-      tmem_ld32(trow + sb * kTileKeys, lo);
-      tmem_ld32(trow + sb * kTileKeys + 32, hi);
+      uint32_t sv[32];
+      tmem_ld32(trow + sbuf * kTileKeys + 32 * wg, sv);
       tmem_wait_ld();
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        sv[j] = lo[j];
-        sv[32 + j] = hi[j];
-      }
-    }
-    if (live && warp_live) {
-      // Visible keys of this row in this tile as a 64-bit mask (bit j = key j of the tile).
-      uint64_t vis = 0;
+      // Visible keys of this row among the warpgroup's 32 columns (bit j = column 32 wg + j).
+      uint32_t vis = 0;
       if (valid) {
-        vis = ti.nkeys >= 64 ? ~0ull : ((1ull << ti.nkeys) - 1ull);
+        uint64_t v64 = ti.nkeys >= 64 ? ~0ull : ((1ull << ti.nkeys) - 1ull);
         if (ti.draft) {
           uint64_t dm;
           if (tree) {
@@ -319,13 +345,14 @@ __device__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pip
             const int last = n_nodes - nq + nl - ti.key0;  // chain: slots key0 .. node are visible
             dm = last >= 63 ? ~0ull : (last < 0 ? 0ull : ((2ull << last) - 1ull));
           }
-          vis &= dm;
+          v64 &= dm;
         }
+        vis = static_cast<uint32_t>(v64 >> (32 * wg));
       }
       float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int j = 0; j < 64; ++j) {
-        pr[j] = ((vis >> j) & 1ull) ? __uint_as_float(sv[j]) * qscale : -INFINITY;
+      for (int j = 0; j < 32; ++j) {
+        pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * qscale : -INFINITY;
         mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
       }
       const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
@@ -333,18 +360,18 @@ __device__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pip
       const bool grow = valid && (m_run == -INFINITY ? mx != -INFINITY : mx > m_run + kRescaleThreshold);
       const bool rescale_o = grow && m_run != -INFINITY;
       if (__any_sync(0xffffffffu, rescale_o)) {
-        // O must hold P.V of the previous tile before it is scaled.
-        if (!mbar_wait(smem_addr(&sm.pvdone[(t - 1) & 1]), ((t - 1) >> 1) & 1, p.err)) *pipe.abort = 1;
+        // O_wg must hold P.V of the previous tile before it is scaled.
+        if (!mbar_wait(smem_addr(&sm.pvdone[(t - 1) % kNP]), ((t - 1) / kNP) & 1, p.err)) *pipe.abort = 1;
         tc_fence_after();
         const float alpha = rescale_o ? ex2(m_run - mx) : 1.f;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           uint32_t o[32];
-          tmem_ld32(trow + kTmemO + 32 * c, o);
+          tmem_ld32(my_o + 32 * c, o);
           tmem_wait_ld();
 #pragma unroll
           for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha);
-          tmem_st32(trow + kTmemO + 32 * c, o);
+          tmem_st32(my_o + 32 * c, o);
         }
         tmem_wait_st();
         l_run *= alpha;
@@ -353,24 +380,25 @@ __device__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pip
       const float m_use = m_run == -INFINITY ? 0.f : m_run;
       float ps4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int j = 0; j < 64; ++j) {
+      for (int j = 0; j < 32; ++j) {
         pr[j] = ex2(pr[j] - m_use);
         ps4[j & 3] += pr[j];
       }
       l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
     }
-    // The P buffer is free once P.V of tile t-2 has completed.
-    if (live && t >= 2 && !mbar_wait(smem_addr(&sm.pvdone[sb]), ((t - 2) >> 1) & 1, p.err)) *pipe.abort = 1;
+    // The P buffer is free once P.V of tile t - kNP has completed.
+    if (live && t >= kNP && !mbar_wait(smem_addr(&sm.pvdone[b]), ((t - kNP) / kNP) & 1, p.err)) *pipe.abort = 1;
     if (live && valid) {
-      uint8_t* prow = sm.pbuf + sb * kPBufBytes + r * 128;
+      uint8_t* prow = sm.pbuf + b * kPBufBytes + r * 128;
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
+      for (int c = 0; c < 4; ++c) {
+        const int chunk = 4 * wg + c;  // 16-byte chunk = 8 keys
         uint4 w;
         w.x = pack_bf16x2(pr[8 * c + 0], pr[8 * c + 1]);
         w.y = pack_bf16x2(pr[8 * c + 2], pr[8 * c + 3]);
         w.z = pack_bf16x2(pr[8 * c + 4], pr[8 * c + 5]);
         w.w = pack_bf16x2(pr[8 * c + 6], pr[8 * c + 7]);
-        *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = w;
+        *reinterpret_cast<uint4*>(prow + ((chunk ^ (r & 7)) << 4)) = w;
       }
     }
     if (live && ti.nkeys < kTileKeys) {
@@ -385,45 +413,59 @@ __device__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pip
     }
     fence_proxy_async_smem();
     tc_fence_before();
-    mbar_arrive(smem_addr(&sm.pfull[sb]));
+    mbar_arrive(smem_addr(&sm.pfull[b]));
     if (ti.last) {
-      bool ok = live && mbar_wait(smem_addr(&sm.pvdone[sb]), (t >> 1) & 1, p.err);
+      bool ok = live && mbar_wait(smem_addr(&sm.pvdone[b]), (t / kNP) & 1, p.err);
       ok = __all_sync(0xffffffffu, ok);
       tc_fence_after();
-      if (ok && warp_live) {
+      // Merge the two warpgroups' states: warpgroup 1 publishes (max, sum), warpgroup 0 writes the row.
+      if (wg == 1) {
+        sm.comb[2 * r] = m_run;
+        sm.comb[2 * r + 1] = l_run;
+      }
+      named_barrier_sync(kBarSoftmax, kSoftmaxThreads);
+      if (wg == 0 && ok && warp_live) {
+        const float m1 = sm.comb[2 * r], l1 = sm.comb[2 * r + 1];
+        const float M = fmaxf(m_run, m1);
+        const float w0 = m_run == -INFINITY ? 0.f : ex2(m_run - M);
+        const float w1 = m1 == -INFINITY ? 0.f : ex2(m1 - M);
+        const float L = w0 * l_run + w1 * l1;
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        const float a0 = w0 * inv, a1 = w1 * inv;
+        const float lse2 = L > 0.f ? M + __log2f(L) : -INFINITY;
         const bool whole = cu.lt == cu.ut - 1 && (cu.t - cu.t_begin) >= cu.lt;
         const int slot = cu.c * HR + cu.hr + blockIdx.x;
-        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-        const float lse2 = l_run > 0.f ? m_run + __log2f(l_run) : -INFINITY;
         size_t orow = 0;
         if (valid && whole) {
           const int g = rr - nl * p.G;
           orow = (static_cast<size_t>(cu.c) * p.Nq + nl) * p.hq + h * p.G + g;
         }
-#pragma unroll
+#pragma unroll 1
         for (int c = 0; c < 4; ++c) {
-          uint32_t o[32];
-          tmem_ld32(trow + kTmemO + 32 * c, o);
+          uint32_t o0[32], o1[32];
+          tmem_ld32(trow + kTmemO + 32 * c, o0);
+          tmem_ld32(trow + kTmemO + 128 + 32 * c, o1);
           tmem_wait_ld();
+          float v[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = a0 * __uint_as_float(o0[j]) + a1 * __uint_as_float(o1[j]);
           if (valid) {
             if (whole) {
               uint4* dst = reinterpret_cast<uint4*>(p.out + orow * kHeadDim + 32 * c);
 #pragma unroll
               for (int k = 0; k < 4; ++k) {
                 uint4 w;
-                w.x = pack_bf16x2(__uint_as_float(o[8 * k + 0]) * inv, __uint_as_float(o[8 * k + 1]) * inv);
-                w.y = pack_bf16x2(__uint_as_float(o[8 * k + 2]) * inv, __uint_as_float(o[8 * k + 3]) * inv);
-                w.z = pack_bf16x2(__uint_as_float(o[8 * k + 4]) * inv, __uint_as_float(o[8 * k + 5]) * inv);
-                w.w = pack_bf16x2(__uint_as_float(o[8 * k + 6]) * inv, __uint_as_float(o[8 * k + 7]) * inv);
+                w.x = pack_bf16x2(v[8 * k + 0], v[8 * k + 1]);
+                w.y = pack_bf16x2(v[8 * k + 2], v[8 * k + 3]);
+                w.z = pack_bf16x2(v[8 * k + 4], v[8 * k + 5]);
+                w.w = pack_bf16x2(v[8 * k + 6], v[8 * k + 7]);
                 dst[k] = w;
               }
             } else {
               float4* dst = reinterpret_cast<float4*>(
                   p.ws_o + (static_cast<size_t>(slot) * p.rows_per_unit + r) * kHeadDim + 32 * c);
 #pragma unroll
-              for (int k = 0; k < 8; ++k)
-                dst[k] = make_float4(__uint_as_float(o[4 * k]) * inv, __uint_as_float(o[4 * k + 1]) * inv,
-                                     __uint_as_float(o[4 * k + 2]) * inv, __uint_as_float(o[4 * k + 3]) * inv);
+              for (int k = 0; k < 8; ++k) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
             }
           }
         }
@@ -432,6 +474,7 @@ __device__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pip
           else p.ws_lse[static_cast<size_t>(slot) * p.rows_per_unit + r] = lse2;
         }
       }
+      named_barrier_sync(kBarSoftmax, kSoftmaxThreads);  // comb is reused at the next piece end
       tc_fence_before();
       mbar_arrive(smem_addr(sm.ofree));
     }
@@ -453,10 +496,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_addr(&sm.full[s]), 1);
       mbar_init(smem_addr(&sm.empty[s]), 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(smem_addr(&sm.qfull[b]), 1);
-      mbar_init(smem_addr(&sm.qempty[b]), 1);
-      mbar_init(smem_addr(&sm.sfull[b]), 1);
+    mbar_init(smem_addr(sm.qfull), 1);
+    mbar_init(smem_addr(sm.qempty), 1);
+    for (int b = 0; b < kNS; ++b) mbar_init(smem_addr(&sm.sfull[b]), 1);
+    for (int b = 0; b < kNP; ++b) {
       mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads);
       mbar_init(smem_addr(&sm.pvdone[b]), 1);
     }
@@ -470,7 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tensormap(&maps.dv);
     prefetch_tensormap(&maps.q);
   }
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tmem_alloc(smem_addr(sm.tmem_base), kTmemCols);
     tmem_relinquish();
   }
@@ -480,17 +523,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *sm.tmem_base;
   const Cursor cu = cursor_begin(p, sm.len, sm.base);
   Pipe pipe{sm.ring, sm.full, sm.empty, kStages, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
-  QPipe qp{sm.qbuf, sm.qfull, sm.qempty, p.G * nq_box, nq_box, &sm.misc[3]};
-  if (warp == 0) {
+  QPipe qp{sm.qbuf, sm.qfull, sm.qempty, 1, p.G * nq_box, nq_box, &sm.misc[3]};
+  if (warp == kProducerWarp) {
     run_producer(p, maps, pipe, sm.len, cu, &qp);
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
       run_mma(p, sm, pipe, tmem, cu);
       // Every MMA must have completed before TMEM is released.
       mbar_wait(smem_addr(sm.mmadone), 0, p.err);
     }
     __syncwarp();
-  } else {
+  } else if (warp < 8) {
     run_softmax(p, sm, pipe, tmem, cu);
   }
   tc_fence_before();
@@ -500,9 +543,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // A wait timed out: let every TMA load still in flight land before the CTA exits.
     drain_after_abort(p, pipe, sm.misc[2]);
     for (int k = sm.misc[4]; k < sm.misc[3]; ++k)
-      if (!mbar_wait(smem_addr(&sm.qfull[k & 1]), (k >> 1) & 1, p.err)) break;
+      if (!mbar_wait(smem_addr(sm.qfull), k & 1, p.err)) break;
   }
-  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+  if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
 }
 
 }  // namespace

@@ -139,12 +139,20 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   const int G = d->hq / d->hkv;
   const int rows = G * d->n_query;
   const bool force_cc = d->flags & KVSHOT_FORCE_CC, force_tc = d->flags & KVSHOT_FORCE_TC;
-  // Measured on GB300 (ncu + bench): at 4 stacked rows the CUDA-core kernel is
-  // issue/latency bound (IPC ~1, ~100 warp instructions per key) while the
-  // m16n8k16 kernel, with the stack zero-padded to 16 rows, streams K/V at
-  // 73-97% of HBM bandwidth; so the tensor-core kernel is the default for every
-  // stack size and the CUDA-core kernel is kept behind KVSHOT_FORCE_CC.
-  pl->kernel = force_cc ? Kernel::kCudaCore : force_tc ? Kernel::kTensorMemory : Kernel::kMma;
+  const bool force_mma = d->flags & KVSHOT_FORCE_MMA;
+  // Kernel choice, measured on GB300 (bench + ncu):
+  //  - up to 16 stacked rows per KV head the m16n8k16 kernel streams K/V at
+  //    90-98% of HBM bandwidth, also at 4 rows where the CUDA-core kernel is
+  //    issue bound (IPC ~1, ~100 warp instructions per key, 23%); the CUDA-core
+  //    kernel stays behind KVSHOT_FORCE_CC;
+  //  - from 17 rows on, the mma.sync kernel becomes latency bound (one warp per
+  //    16-row tile) and the tcgen05 kernel, whose MMAs run asynchronously out of
+  //    shared memory into tensor memory, is faster (1.5x at 48 rows, 3-4x for
+  //    whole-tree stacks of 128-256 rows).
+  const bool tc_ok = G <= 128 && 128 % G == 0;
+  const Kernel automatic = (rows > 16 && tc_ok) ? Kernel::kTensorMemory : Kernel::kMma;
+  pl->kernel = force_cc ? Kernel::kCudaCore : force_tc ? Kernel::kTensorMemory
+                                           : force_mma ? Kernel::kMma : automatic;
   pl->mma = pl->kernel == Kernel::kMma;
   pl->m_tiles = 0;
   pl->nq_box = 0;

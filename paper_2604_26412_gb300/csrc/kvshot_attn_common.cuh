@@ -80,6 +80,19 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t
   return mbar_wait_slow(bar, parity, err);
 }
 
+// Non-blocking test of a phase's completion.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(done)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
 __device__ __forceinline__ uint64_t l2_policy_evict_first() {
   uint64_t pol;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
@@ -182,7 +195,7 @@ __device__ __forceinline__ int clamp_len(const AttnParams& p, int c) {
 // s_len[c] = clamped L_c; s_base[c] = first global tile of cache c (prefix sum of
 // units x tiles per unit).  Whole block participates.  CTA 0 also publishes
 // s_base to the workspace for the merge kernel.
-__device__ void build_plan(const AttnParams& p, int* s_len, int* s_base) {
+__device__ __forceinline__ void build_plan(const AttnParams& p, int* s_len, int* s_base) {
   const int HR = p.hkv * p.row_blocks;
   for (int c = threadIdx.x; c < p.C; c += blockDim.x) {
     const int L = clamp_len(p, c);
@@ -226,7 +239,7 @@ __device__ __forceinline__ void cursor_load_cache(Cursor& cu, const AttnParams& 
   cu.ut = cu.pt + p.draft_tiles;
 }
 
-__device__ Cursor cursor_begin(const AttnParams& p, const int* s_len, const int* s_base) {
+__device__ __forceinline__ Cursor cursor_begin(const AttnParams& p, const int* s_len, const int* s_base) {
   Cursor cu;
   const int total = s_base[p.C];
   const int tpc = tiles_per_cta(total, p.num_ctas);
@@ -288,7 +301,7 @@ __device__ __forceinline__ TileInfo tile_info(const Cursor& cu, const AttnParams
 // `nthreads` consumer threads (tid in [0, nthreads)), which must all call it;
 // two named barriers (id `bar`) fence it.  Invalid parents are reported and
 // treated as roots.
-__device__ void build_ancestor_masks(const AttnParams& p, int seq, uint64_t* s_anc, int* s_par, int tid,
+__device__ __forceinline__ void build_ancestor_masks(const AttnParams& p, int seq, uint64_t* s_anc, int* s_par, int tid,
                                      int nthreads, int bar) {
   const int* par = p.tree_parent + static_cast<size_t>(seq) * p.N;
   for (int i = tid; i < p.N; i += nthreads) {
@@ -348,12 +361,13 @@ struct Pipe {
   int* issued;         // tiles issued by the producer
 };
 
-// Double-buffered q staging (tensor-memory kernel only): piece k's query
-// block goes to buffer k % 2 (two 64-dim halves of 128 rows, 128B-swizzled).
+// q staging (tensor-memory kernel only): piece k's query block goes to buffer
+// k % nbuf (two 64-dim halves of 128 rows, 128B-swizzled).
 struct QPipe {
-  uint8_t* buf;        // 2 x kQBufBytes, 1024-aligned
-  uint64_t* full;      // [2] TMA -> MMA issuer
-  uint64_t* empty;     // [2] MMA completion -> TMA
+  uint8_t* buf;        // nbuf x kQBufBytes, 1024-aligned
+  uint64_t* full;      // [nbuf] TMA -> MMA issuer
+  uint64_t* empty;     // [nbuf] MMA completion -> TMA
+  int nbuf;            // q buffers (piece k uses buffer k % nbuf)
   int rows;            // rows loaded per box (G x nodes per box)
   int nq_box;          // draft nodes per box
   int* issued;         // q blocks issued
@@ -363,7 +377,7 @@ constexpr int kQBufBytes = 2 * kQRows * 128;
 
 // The producer warp: walks this CTA's tiles and issues their TMA loads into the
 // stage ring, one tile ahead on the page-table reads.  Lane 0 issues.
-__device__ void run_producer(const AttnParams& p, const TensorMaps& maps, const Pipe& pipe, const int* s_len,
+__device__ __forceinline__ void run_producer(const AttnParams& p, const TensorMaps& maps, const Pipe& pipe, const int* s_len,
                              Cursor cu, const QPipe* qp = nullptr) {
   const int lane = threadIdx.x & 31;
   const uint64_t policy = l2_policy_evict_first();
@@ -392,9 +406,9 @@ __device__ void run_producer(const AttnParams& p, const TensorMaps& maps, const 
     if (qp != nullptr && (cu.t == cu.t_begin || cu.lt == 0)) {
       // First tile of a piece: stage the unit's query block (all its G x Nq rows).
       if (lane == 0) {
-        const int qb = piece & 1;
+        const int qb = piece % qp->nbuf;
         const uint32_t qbar = smem_addr(&qp->full[qb]);
-        ok = mbar_wait(smem_addr(&qp->empty[qb]), ((piece >> 1) & 1) ^ 1u, p.err) ? 1 : 0;
+        ok = mbar_wait(smem_addr(&qp->empty[qb]), ((piece / qp->nbuf) & 1) ^ 1u, p.err) ? 1 : 0;
         if (ok && !*pipe.abort) {
           const int rb = cu.hr - h * p.row_blocks;
           const uint32_t dst = smem_addr(qp->buf + qb * kQBufBytes);
@@ -417,46 +431,39 @@ __device__ void run_producer(const AttnParams& p, const TensorMaps& maps, const 
       if (lane == 0) *pipe.abort = 1;
       break;
     }
-    if (lane == 0) {
+    {
+      // Lane 0 posts the tile's byte count; every lane then issues at most one
+      // box: box = lane -> (tensor K/V, 64-dim half, page or 8-row group).
       const uint32_t full_bar = smem_addr(&pipe.full[stage]);
       const uint32_t kdst = smem_addr(pipe.ring + static_cast<size_t>(stage) * kStageBytes);
-      const uint32_t vdst = kdst + kKVTileBytes;
+      const int kv = lane & 1, hf = (lane >> 1) & 1, i = lane >> 2;
+      const uint32_t dst = kdst + kv * kKVTileBytes + hf * kHalfBytes;
       if (draft) {
         const int nbox = (nkeys + kDraftBoxRows - 1) / kDraftBoxRows;
-        mbar_arrive_expect_tx(full_bar, nbox * kDraftBoxRows * 128 * 4);
-        const int y0 = (cu.c * p.hkv + h) * p.n_max + key0;
-        for (int i = 0; i < nbox; ++i) {
-          const uint32_t off = i * kDraftBoxRows * 128;
-#pragma unroll
-          for (int hf = 0; hf < 2; ++hf) {
-            tma_load_2d(kdst + hf * kHalfBytes + off, &maps.dk, hf * 64, y0 + i * kDraftBoxRows, full_bar, policy);
-            tma_load_2d(vdst + hf * kHalfBytes + off, &maps.dv, hf * 64, y0 + i * kDraftBoxRows, full_bar, policy);
-          }
+        if (lane == 0) mbar_arrive_expect_tx(full_bar, nbox * kDraftBoxRows * 128 * 4);
+        if (i < nbox) {
+          const int y0 = (cu.c * p.hkv + h) * p.n_max + key0;
+          tma_load_2d(dst + i * kDraftBoxRows * 128, kv ? &maps.dv : &maps.dk, hf * 64, y0 + i * kDraftBoxRows,
+                      full_bar, policy);
         }
       } else if (p.paged) {
         const int br = p.box_rows;
         const int nbox = (nkeys + br - 1) / br;
-        mbar_arrive_expect_tx(full_bar, nbox * br * 128 * 4);
+        if (lane == 0) mbar_arrive_expect_tx(full_bar, nbox * br * 128 * 4);
+        if (i < nbox) {
+          int pid = pids[0];
 #pragma unroll
-        for (int i = 0; i < kTileKeys / 8; ++i) {  // box_rows >= 8, so at most 8 boxes
-          if (i < nbox) {
-            const int krow = key0 + i * br;
-            const int y = (pids[i] * p.hkv + h) * p.page_size + (krow % p.page_size);
-            const uint32_t off = i * br * 128;
-#pragma unroll
-            for (int hf = 0; hf < 2; ++hf) {
-              tma_load_2d(kdst + hf * kHalfBytes + off, &maps.tk, hf * 64, y, full_bar, policy);
-              tma_load_2d(vdst + hf * kHalfBytes + off, &maps.tv, hf * 64, y, full_bar, policy);
-            }
-          }
+          for (int k = 1; k < kTileKeys / 8; ++k)
+            if (i == k) pid = pids[k];
+          const int krow = key0 + i * br;
+          const int y = (pid * p.hkv + h) * p.page_size + (krow % p.page_size);
+          tma_load_2d(dst + i * br * 128, kv ? &maps.tv : &maps.tk, hf * 64, y, full_bar, policy);
         }
       } else {
-        mbar_arrive_expect_tx(full_bar, kTileKeys * 128 * 4);
-        const int y = (cu.c * p.hkv + h) * p.l_cap + key0;
-#pragma unroll
-        for (int hf = 0; hf < 2; ++hf) {
-          tma_load_2d(kdst + hf * kHalfBytes, &maps.tk, hf * 64, y, full_bar, policy);
-          tma_load_2d(vdst + hf * kHalfBytes, &maps.tv, hf * 64, y, full_bar, policy);
+        if (lane == 0) mbar_arrive_expect_tx(full_bar, kTileKeys * 128 * 4);
+        if (i == 0) {
+          const int y = (cu.c * p.hkv + h) * p.l_cap + key0;
+          tma_load_2d(dst, kv ? &maps.tv : &maps.tk, hf * 64, y, full_bar, policy);
         }
       }
     }
@@ -474,7 +481,7 @@ __device__ void run_producer(const AttnParams& p, const TensorMaps& maps, const 
 // After the roles finish: if a wait timed out, wait (bounded) for every TMA
 // load still in flight so no copy lands in shared memory after the CTA exits.
 // Called by one thread after a block-wide barrier.
-__device__ void drain_after_abort(const AttnParams& p, const Pipe& pipe, int consumed) {
+__device__ __forceinline__ void drain_after_abort(const AttnParams& p, const Pipe& pipe, int consumed) {
   if (!*pipe.abort) return;
   for (int k = consumed; k < *pipe.issued; ++k) {
     const int st = k % pipe.stages;

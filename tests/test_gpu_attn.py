@@ -76,7 +76,7 @@ def test_attn_matches_oracle(case):
     spec, inp, dk, dv, q, N, Nq = _case(lens, levels, tree, paged, P, hq, hkv, nq, seed=len(lens) + N_SEED(case))
     hc = gh.HostCache(inp)
     ref_out, ref_lse = gh.oracle_attn(hc, q, dk, dv, N, Nq)
-    kernels = [0, kvshot.KVSHOT_FORCE_TC] if 128 % (hq // hkv) == 0 else [0]
+    kernels = [0, kvshot.KVSHOT_FORCE_MMA] + ([kvshot.KVSHOT_FORCE_TC] if 128 % (hq // hkv) == 0 else [])
     for flags in kernels:
         for num_ctas in (0, 1, 7):
             out, lse = _run(spec, inp, dk, dv, q, N, Nq, flags=flags, num_ctas=num_ctas)
@@ -114,7 +114,7 @@ def test_deterministic_across_runs():
     assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
 
 
-@pytest.mark.parametrize("flags", [0, kvshot.KVSHOT_FORCE_TC])
+@pytest.mark.parametrize("flags", [0, kvshot.KVSHOT_FORCE_MMA, kvshot.KVSHOT_FORCE_TC])
 @pytest.mark.parametrize("paged", [False, True])
 @pytest.mark.parametrize("tree", [False, True])
 def test_mask_probe_is_exact(paged, tree, flags):
