@@ -26,7 +26,9 @@ namespace {
 
 using namespace dev;
 
-constexpr int kStages = 4;                 // K/V ring
+constexpr int kNK = 3;                     // K tiles in flight (freed when QK^T completes)
+constexpr int kNV = 5;                     // V tiles in flight (freed when P.V completes)
+constexpr int kKVBytes = kKVTileBytes;     // one K or V tile
 constexpr int kNS = 4;                     // S buffers in TMEM: QK^T may run up to 4 tiles ahead of P.V
 constexpr int kNP = 3;                     // P buffers in shared memory
 constexpr int kThreads = 12 * 32;
@@ -120,11 +122,14 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major)
 // ------------------------------------------------------------ shared memory
 
 struct Smem {
-  uint8_t* ring;       // kStages x (K tile | V tile)
+  uint8_t* kring;      // kNK x K tile
+  uint8_t* vring;      // kNV x V tile
   uint8_t* qbuf;       // one q block
   uint8_t* pbuf;       // kNP x kPBufBytes
-  uint64_t* full;      // [kStages]
-  uint64_t* empty;     // [kStages]  (MMA completion)
+  uint64_t* kfull;     // [kNK]  TMA -> MMA
+  uint64_t* kempty;    // [kNK]  QK^T completion -> TMA
+  uint64_t* vfull;     // [kNV]  TMA -> MMA, softmax
+  uint64_t* vempty;    // [kNV]  P.V completion -> TMA
   uint64_t* qfull;     // [1]
   uint64_t* qempty;    // [1]
   uint64_t* sfull;     // [kNS]  S buffer written (MMA completion)
@@ -136,14 +141,14 @@ struct Smem {
   int* par;            // [64]
   float* comb;         // [128][2] second warpgroup's (max, sum) per row at a piece end
   uint32_t* tmem_base;
-  int* misc;           // [0] abort, [1] tiles issued, [2] tiles consumed, [3] q blocks issued, [4] q consumed
+  int* misc;           // [0] abort, [1]/[2] K tiles issued/consumed, [3]/[4] q blocks, [5]/[6] V tiles
   int* len;
   int* base;
 };
 
 __host__ __device__ inline size_t smem_bytes(int C) {
-  size_t off = static_cast<size_t>(kStages) * kStageBytes + kQBufBytes + kNP * kPBufBytes;
-  off += sizeof(uint64_t) * (2 * kStages + 2 + kNS + 2 * kNP + 2);
+  size_t off = static_cast<size_t>(kNK + kNV) * kKVBytes + kQBufBytes + kNP * kPBufBytes;
+  off += sizeof(uint64_t) * (2 * kNK + 2 * kNV + 2 + kNS + 2 * kNP + 2);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(float) * 2 * kQRows;
   off += sizeof(uint32_t) * 4 + sizeof(int) * 8;
@@ -154,16 +159,20 @@ __host__ __device__ inline size_t smem_bytes(int C) {
 __device__ Smem carve(uint8_t* raw, int C) {
   Smem s;
   uint8_t* p = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
-  s.ring = p;
-  p += kStages * kStageBytes;
+  s.kring = p;
+  p += kNK * kKVBytes;
+  s.vring = p;
+  p += kNV * kKVBytes;
   s.qbuf = p;
   p += kQBufBytes;
   s.pbuf = p;
   p += kNP * kPBufBytes;
   uint64_t* b = reinterpret_cast<uint64_t*>(p);
-  s.full = b;
-  s.empty = s.full + kStages;
-  s.qfull = s.empty + kStages;
+  s.kfull = b;
+  s.kempty = s.kfull + kNK;
+  s.vfull = s.kempty + kNK;
+  s.vempty = s.vfull + kNV;
+  s.qfull = s.vempty + kNV;
   s.qempty = s.qfull + 1;
   s.sfull = s.qempty + 1;
   s.pfull = s.sfull + kNS;
@@ -183,12 +192,13 @@ __device__ Smem carve(uint8_t* raw, int C) {
 // ------------------------------------------------------------ MMA issuer
 
 struct PendingPV {
-  int stage, tile, piece;
+  int tile, piece;
   bool first;
 };
 
 // O_w += P[:, 32w..32w+32) V[32w..32w+32, :] for both warpgroups w.
 __device__ __forceinline__ bool pv_ready(const Smem& sm, const PendingPV& pv) {
+  if (!mbar_test_wait(smem_addr(&sm.vfull[pv.tile % kNV]), (pv.tile / kNV) & 1)) return false;
   if (!mbar_test_wait(smem_addr(&sm.pfull[pv.tile % kNP]), (pv.tile / kNP) & 1)) return false;
   return !(pv.first && pv.piece > 0) || mbar_test_wait(smem_addr(sm.ofree), (pv.piece - 1) & 1);
 }
@@ -198,7 +208,7 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, const Pe
   tc_fence_after();
   constexpr uint32_t idesc = idesc_bf16(128, 128, true);
   const uint32_t pbase = smem_addr(sm.pbuf + b * kPBufBytes);
-  const uint32_t vbase = smem_addr(sm.ring + static_cast<size_t>(pv.stage) * kStageBytes + kKVTileBytes);
+  const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(pv.tile % kNV) * kKVBytes);
 #pragma unroll
   for (int w = 0; w < 2; ++w)
 #pragma unroll
@@ -209,7 +219,7 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, const Pe
       const uint64_t bd = smem_desc_sw128(vbase + k16 * 2048, kHalfBytes, 1024);
       tc_mma(tmem + kTmemO + 128 * w, a, bd, idesc, (pv.first && kk == 0) ? 0u : 1u);
     }
-  tc_commit(smem_addr(&sm.empty[pv.stage]));
+  tc_commit(smem_addr(&sm.vempty[pv.tile % kNV]));
   tc_commit(smem_addr(&sm.pvdone[b]));
 }
 
@@ -219,8 +229,7 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, const Pe
 __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                         Cursor cu) {
   constexpr uint32_t idesc = idesc_bf16(128, 64, false);
-  int stage = 0, next_qk = 0, next_pv = 0, piece = 0, cur_piece = 0;
-  uint32_t phase = 0;
+  int next_qk = 0, next_pv = 0, piece = 0, cur_piece = 0;
   bool q_ready = false;  // the q block of the tile at the cursor is resident
   PendingPV pend[kNS];
   uint64_t idle_since = 0;
@@ -230,7 +239,7 @@ __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, con
     if (cu.t < cu.t_end && next_qk - next_pv < kNS) {
       const TileInfo ti = tile_info(cu, p);
       if (ti.first && !q_ready) q_ready = mbar_test_wait(smem_addr(sm.qfull), piece & 1);
-      if ((!ti.first || q_ready) && mbar_test_wait(smem_addr(&pipe.full[stage]), phase)) {
+      if ((!ti.first || q_ready) && mbar_test_wait(smem_addr(&sm.kfull[next_qk % kNK]), (next_qk / kNK) & 1)) {
         if (ti.first) {
           cur_piece = piece++;
           sm.misc[4] = piece;
@@ -239,7 +248,7 @@ __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, con
         sm.misc[2] = next_qk + 1;
         tc_fence_after();
         const uint32_t qbase = smem_addr(sm.qbuf);
-        const uint32_t kbase = smem_addr(sm.ring + static_cast<size_t>(stage) * kStageBytes);
+        const uint32_t kbase = smem_addr(sm.kring + static_cast<size_t>(next_qk % kNK) * kKVBytes);
 #pragma unroll
         for (int ks = 0; ks < kHeadDim / 16; ++ks) {
           const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
@@ -247,13 +256,10 @@ __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, con
           tc_mma(tmem + (next_qk % kNS) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
         }
         tc_commit(smem_addr(&sm.sfull[next_qk % kNS]));
+        tc_commit(smem_addr(&sm.kempty[next_qk % kNK]));
         if (ti.last) tc_commit(smem_addr(sm.qempty));
-        pend[next_qk % kNS] = PendingPV{stage, next_qk, cur_piece, ti.first};
+        pend[next_qk % kNS] = PendingPV{next_qk, cur_piece, ti.first};
         ++next_qk;
-        if (++stage == kStages) {
-          stage = 0;
-          phase ^= 1u;
-        }
         cursor_next(cu, p, sm.len);
         progressed = true;
       }
@@ -261,6 +267,7 @@ __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, con
     if (next_pv < next_qk && pv_ready(sm, pend[next_pv % kNS])) {
       issue_pv(sm, tmem, pend[next_pv % kNS]);
       ++next_pv;
+      sm.misc[6] = next_pv;
       progressed = true;
     }
     if (cu.t >= cu.t_end && next_pv == next_qk) break;
@@ -299,8 +306,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
   const bool tree = p.tree != 0;
   const int nq = p.Nq, n_nodes = p.N;
   float m_run = -INFINITY, l_run = 0.f;
-  int t = 0, stage = 0, anc_seq = -1;
-  uint32_t phase = 0;
+  int t = 0, anc_seq = -1;
   for (; cu.t < cu.t_end; cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
     const int h = cu.hr / p.row_blocks, rb = cu.hr - h * p.row_blocks;
@@ -403,8 +409,8 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
     }
     if (live && ti.nkeys < kTileKeys) {
       // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.
-      if (!mbar_wait(smem_addr(&pipe.full[stage]), phase, p.err)) *pipe.abort = 1;
-      uint8_t* vptr = pipe.ring + static_cast<size_t>(stage) * kStageBytes + kKVTileBytes;
+      if (!mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err)) *pipe.abort = 1;
+      uint8_t* vptr = sm.vring + static_cast<size_t>(t % kNV) * kKVBytes;
       const int nz = (kTileKeys - ti.nkeys) * 16;
       for (int i = tid; i < nz; i += kSoftmaxThreads) {
         const int key = ti.nkeys + (i >> 4), ch = i & 15;
@@ -479,10 +485,89 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       mbar_arrive(smem_addr(sm.ofree));
     }
     ++t;
-    if (++stage == kStages) {
-      stage = 0;
-      phase ^= 1u;
+  }
+}
+
+// ------------------------------------------------------------ TMA producer
+
+// Walks this CTA's tiles: one q block per piece (single buffer), the K tile
+// into the K ring and the V tile into the V ring, each box from its own lane.
+__device__ __forceinline__ void run_producer_tc(const AttnParams& p, const TensorMaps& maps, const Smem& sm,
+                                                const Pipe& pipe, Cursor cu, int nq_box) {
+  const int lane = threadIdx.x & 31;
+  const uint64_t policy = l2_policy_evict_first();
+  PageWindow win;
+  int t = 0, piece = 0;
+  const int rows_q = p.G * nq_box;
+  while (cu.t < cu.t_end) {
+    const int h = cu.hr / p.row_blocks;
+    const bool draft = cu.lt >= cu.pt;
+    const int key0 = (draft ? cu.lt - cu.pt : cu.lt) * kTileKeys;
+    const int nkeys = min(kTileKeys, (draft ? p.N : cu.L) - key0);
+    int pid = 0;  // page id of this lane's box
+    int nbox, br;
+    if (draft) {
+      br = kDraftBoxRows;
+      nbox = (nkeys + br - 1) / br;
+    } else if (p.paged) {
+      br = p.box_rows;
+      nbox = (nkeys + br - 1) / br;
+      const int pg0 = key0 / p.page_size;
+      const int npg = br < p.page_size ? 1 : nbox;
+      win.cover(p, cu.c, (cu.L + p.page_size - 1) / p.page_size, pg0, npg, lane);
+      const int i = min(lane >> 1, npg - 1);
+      pid = win.get(pg0 + (br < p.page_size ? 0 : i));
+    } else {
+      br = kTileKeys;
+      nbox = 1;
     }
+    const int hf = lane & 1, i = lane >> 1;  // this lane's box: 64-dim half, row group
+    int y = 0;
+    if (draft) y = (cu.c * p.hkv + h) * p.n_max + key0 + i * br;
+    else if (p.paged) y = (pid * p.hkv + h) * p.page_size + ((key0 + i * br) % p.page_size);
+    else y = (cu.c * p.hkv + h) * p.l_cap + key0;
+    const uint32_t tx = nbox * br * 128 * 2;  // bytes of one K (or V) tile's boxes
+    int ok = 1;
+    if (cu.t == cu.t_begin || cu.lt == 0) {  // first tile of a piece: the unit's q block
+      if (lane == 0) {
+        const uint32_t qbar = smem_addr(sm.qfull);
+        ok = mbar_wait(smem_addr(sm.qempty), (piece & 1) ^ 1u, p.err) && !*pipe.abort;
+        if (ok) {
+          const int rb = cu.hr - h * p.row_blocks;
+          const uint32_t dst = smem_addr(sm.qbuf);
+          mbar_arrive_expect_tx(qbar, 2 * rows_q * 128);
+          tma_load_4d(dst, &maps.q, 0, h * p.G, rb * nq_box, cu.c, qbar);
+          tma_load_4d(dst + kQRows * 128, &maps.q, 64, h * p.G, rb * nq_box, cu.c, qbar);
+          sm.misc[3] = piece + 1;
+        }
+      }
+      ++piece;
+    }
+#pragma unroll
+    for (int kv = 0; kv < 2; ++kv) {
+      const int slot = kv ? t % kNV : t % kNK;
+      const int round = kv ? t / kNV : t / kNK;
+      uint64_t* fullb = kv ? &sm.vfull[slot] : &sm.kfull[slot];
+      uint64_t* emptyb = kv ? &sm.vempty[slot] : &sm.kempty[slot];
+      if (lane == 0 && ok) ok = mbar_wait(smem_addr(emptyb), (round & 1) ^ 1u, p.err) && !*pipe.abort;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      const uint32_t full_bar = smem_addr(fullb);
+      if (lane == 0) mbar_arrive_expect_tx(full_bar, tx);
+      if (i < nbox) {
+        const uint32_t dst = smem_addr((kv ? sm.vring : sm.kring) + static_cast<size_t>(slot) * kKVBytes) +
+                             hf * kHalfBytes + i * br * 128;
+        const CUtensorMap* map = draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
+        tma_load_2d(dst, map, hf * 64, y, full_bar, policy);
+      }
+      if (lane == 0) sm.misc[kv ? 5 : 1] = t + 1;
+    }
+    if (!ok) {
+      if (lane == 0) *pipe.abort = 1;
+      break;
+    }
+    ++t;
+    cursor_next(cu, p, sm.len);
   }
 }
 
@@ -492,9 +577,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const Smem sm = carve(smem_raw, p.C);
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(smem_addr(&sm.full[s]), 1);
-      mbar_init(smem_addr(&sm.empty[s]), 1);
+    for (int s = 0; s < kNK; ++s) {
+      mbar_init(smem_addr(&sm.kfull[s]), 1);
+      mbar_init(smem_addr(&sm.kempty[s]), 1);
+    }
+    for (int s = 0; s < kNV; ++s) {
+      mbar_init(smem_addr(&sm.vfull[s]), 1);
+      mbar_init(smem_addr(&sm.vempty[s]), 1);
     }
     mbar_init(smem_addr(sm.qfull), 1);
     mbar_init(smem_addr(sm.qempty), 1);
@@ -522,10 +611,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *sm.tmem_base;
   const Cursor cu = cursor_begin(p, sm.len, sm.base);
-  Pipe pipe{sm.ring, sm.full, sm.empty, kStages, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
-  QPipe qp{sm.qbuf, sm.qfull, sm.qempty, 1, p.G * nq_box, nq_box, &sm.misc[3]};
+  Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
   if (warp == kProducerWarp) {
-    run_producer(p, maps, pipe, sm.len, cu, &qp);
+    run_producer_tc(p, maps, sm, pipe, cu, nq_box);
   } else if (warp == kMmaWarp) {
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
       run_mma(p, sm, pipe, tmem, cu);
@@ -541,7 +629,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   if (threadIdx.x == 0 && *pipe.abort) {
     // A wait timed out: let every TMA load still in flight land before the CTA exits.
-    drain_after_abort(p, pipe, sm.misc[2]);
+    for (int k = sm.misc[2]; k < sm.misc[1]; ++k)
+      if (!mbar_wait(smem_addr(&sm.kfull[k % kNK]), (k / kNK) & 1, p.err)) break;
+    for (int k = sm.misc[6]; k < sm.misc[5]; ++k)
+      if (!mbar_wait(smem_addr(&sm.vfull[k % kNV]), (k / kNV) & 1, p.err)) break;
     for (int k = sm.misc[4]; k < sm.misc[3]; ++k)
       if (!mbar_wait(smem_addr(sm.qfull), k & 1, p.err)) break;
   }

@@ -331,18 +331,6 @@ __device__ __forceinline__ bool draft_visible(const AttnParams& p, const uint64_
 
 // ------------------------------------------------------------ TMA producer
 
-// Raw (unvalidated) lane-distributed page ids of a paged prefix tile: lane i
-// holds box i's page.  Validation happens at use time (valid_page_id), so the
-// load stays in flight while the producer waits for a free stage.
-__device__ __forceinline__ int tile_page_ids(const AttnParams& p, const Cursor& cu, int lane) {
-  if (cu.t >= cu.t_end || !p.paged || cu.lt >= cu.pt) return 0;
-  const int key0 = cu.lt * kTileKeys;
-  const int nkeys = min(kTileKeys, cu.L - key0);
-  const int nbox = (nkeys + p.box_rows - 1) / p.box_rows;
-  if (lane >= nbox) return 0;
-  return p.page_table[static_cast<size_t>(cu.c) * p.max_pages + (key0 + lane * p.box_rows) / p.page_size];
-}
-
 // A page id checked against the pool; out-of-range ids are reported and replaced by page 0.
 __device__ __forceinline__ int valid_page_id(const AttnParams& p, int pid) {
   if (pid < 0 || pid >= p.num_pages) {
@@ -351,6 +339,51 @@ __device__ __forceinline__ int valid_page_id(const AttnParams& p, int pid) {
   }
   return pid;
 }
+
+// Page ids of the producer warp, 32 consecutive page-table entries of one
+// cache per load (lane i holds entry base + i, validated when loaded),
+// double-buffered: while the current window is used the next one is already
+// in flight.  The cache's first window is kept as well, since the KV heads of
+// one cache (consecutive units) walk the same pages.
+struct PageWindow {
+  int cur_c = -1, cur_base = 0, cur_pid = 0;
+  int nxt_c = -1, nxt_base = 0, nxt_pid = 0;
+  int head_c = -1, head_pid = 0;
+
+  __device__ __forceinline__ static int load(const AttnParams& p, int c, int base, int lane) {
+    const int pg = base + lane;
+    return pg < p.max_pages ? p.page_table[static_cast<size_t>(c) * p.max_pages + pg] : 0;
+  }
+  // Make pages [pg, pg + n) of cache c (n <= 32, windows stay aligned to the
+  // tile's page count; the cache has `pages` pages in use) available in
+  // cur_pid.  Only entries of pages in use are validated.  Warp-wide.
+  __device__ __forceinline__ void cover(const AttnParams& p, int c, int pages, int pg, int n, int lane) {
+    if (cur_c == c && pg >= cur_base && pg + n <= cur_base + 32) return;
+    if (nxt_c == c && pg >= nxt_base && pg + n <= nxt_base + 32) {
+      cur_c = nxt_c;
+      cur_base = nxt_base;
+      cur_pid = nxt_base + lane < pages ? valid_page_id(p, nxt_pid) : 0;
+    } else if (pg == 0 && head_c == c) {
+      cur_c = c;
+      cur_base = 0;
+      cur_pid = head_pid;
+    } else {
+      cur_c = c;
+      cur_base = pg;
+      cur_pid = load(p, c, pg, lane);
+      cur_pid = pg + lane < pages ? valid_page_id(p, cur_pid) : 0;
+      if (pg == 0) {
+        head_c = c;
+        head_pid = cur_pid;
+      }
+    }
+    nxt_c = c;
+    nxt_base = cur_base + 32;
+    nxt_pid = load(p, c, nxt_base, lane);  // validated when it becomes current
+  }
+  // Page id of page pg (covered), broadcast to the warp.
+  __device__ __forceinline__ int get(int pg) const { return __shfl_sync(0xffffffffu, cur_pid, pg - cur_base); }
+};
 
 struct Pipe {
   uint8_t* ring;       // stages x kStageBytes, 1024-aligned
@@ -385,22 +418,23 @@ __device__ __forceinline__ void run_producer(const AttnParams& p, const TensorMa
   uint32_t phase = 0;
   int issued = 0;
   int piece = 0;
-  int pid_cur = tile_page_ids(p, cu, lane);
+  PageWindow win;
   while (cu.t < cu.t_end) {
-    Cursor nx = cu;
-    cursor_next(nx, p, s_len);
-    const int pid_next = tile_page_ids(p, nx, lane);  // in flight while we wait for a free stage
-
     const int h = cu.hr / p.row_blocks;
     const int L = cu.L;
     const bool draft = cu.lt >= cu.pt;
     const int key0 = (draft ? cu.lt - cu.pt : cu.lt) * kTileKeys;
     const int nkeys = min(kTileKeys, (draft ? p.N : L) - key0);
-    // Lane-distributed ids -> lane 0 (shuffles are warp-wide).
+    // Page ids of this tile's boxes (box i covers rows key0 + i * box_rows).
     int pids[kTileKeys / 8];
-    if (p.paged && !draft) pid_cur = valid_page_id(p, pid_cur);
+    if (p.paged && !draft) {
+      const int pg0 = key0 / p.page_size;
+      const int npg = (nkeys + p.box_rows - 1) / p.box_rows;  // one box per page (or one box inside a page)
+      win.cover(p, cu.c, (cu.L + p.page_size - 1) / p.page_size, pg0, p.box_rows < p.page_size ? 1 : npg, lane);
 #pragma unroll
-    for (int i = 0; i < kTileKeys / 8; ++i) pids[i] = __shfl_sync(0xffffffffu, pid_cur, i);
+      for (int i = 0; i < kTileKeys / 8; ++i)
+        pids[i] = win.get(pg0 + (p.box_rows < p.page_size ? 0 : min(i, npg - 1)));
+    }
 
     int ok = 1;
     if (qp != nullptr && (cu.t == cu.t_begin || cu.lt == 0)) {
@@ -468,8 +502,7 @@ __device__ __forceinline__ void run_producer(const AttnParams& p, const TensorMa
       }
     }
     ++issued;
-    pid_cur = pid_next;
-    cu = nx;
+    cursor_next(cu, p, s_len);
     if (++stage == pipe.stages) {
       stage = 0;
       phase ^= 1u;
