@@ -7,18 +7,18 @@
 //   S = Q K^T      tcgen05.mma M=128 N=64  K=128 (8 x K16), A = Q (smem), B = K tile (smem), D = S (TMEM)
 //   P = softmax(S) one thread per row: TMEM -> registers -> bf16 P (smem, 128B-swizzled)
 //   O += P V       tcgen05.mma M=128 N=128 K=64 (4 x K16), A = P (smem), B = V tile (smem, MN-major), D = O (TMEM)
-// Warp roles: warps 0..7 are two softmax warpgroups, warp 10 issues TMA
-// (K/V tiles, one q block per piece), warp 11 owns TMEM and one of its
-// threads issues every MMA (warps 8, 9 idle).  A warp issues from SM
-// sub-partition warp % 4; the TMA and MMA warps sit on sub-partitions 2 and 3,
-// away from the rows 0..31 softmax warps that small GQA stacks keep busiest.  Warpgroup w takes key columns [32w, 32w+32) of every
-// tile with its own running max/sum and its own O accumulator O_w in TMEM
-// (thread = TMEM lane = row); the two are merged by log-sum-exp at the end of
-// each piece.  S has four TMEM buffers; the MMA thread issues QK^T as soon as
-// a K tile and an S buffer are free and P.V as soon as P is written, so QK^T
-// runs ahead of the softmax and the in-order MMA latency hides behind it.  O_w is rescaled in TMEM only
-// when a row's running max grows by more than 2^8 (lazy rescale).  Rows of
-// the 128-row MMA beyond the unit's stack carry no output.
+// Warp roles: warps 0..7 are two softmax warpgroups; warp 10 loads K tiles
+// and the q block of each piece by TMA, warp 9 loads V tiles (a single warp
+// keeps too few bulk-tensor loads in flight to reach full HBM bandwidth);
+// warp 11 owns TMEM and one of its threads issues every MMA (warp 8 idles).
+// Warpgroup w owns the tiles t with t % 2 == w: it turns S into P for all 64
+// keys with its own running max/sum and its own O accumulator O_w in TMEM, so
+// the two warpgroups' per-tile chains overlap; the states are merged by
+// log-sum-exp at the end of each piece.  S has four TMEM buffers; the MMA
+// thread issues QK^T as soon as a K tile and an S buffer are free and P.V as
+// soon as P is written, so QK^T runs ahead of the softmax.  O_w is rescaled in
+// TMEM only when a row's running max grows by more than 2^8 (lazy rescale).
+// Rows of the 128-row MMA that hold no stacked row carry no output.
 #include "kvshot_attn_common.cuh"
 
 namespace kvshot {
@@ -32,7 +32,8 @@ constexpr int kKVBytes = kKVTileBytes;     // one K or V tile
 constexpr int kNS = 4;                     // S buffers in TMEM: QK^T may run up to 4 tiles ahead of P.V
 constexpr int kNP = 3;                     // P buffers in shared memory
 constexpr int kThreads = 12 * 32;
-constexpr int kProducerWarp = 10;
+constexpr int kProducerWarp = 10;          // K ring and q blocks
+constexpr int kProducerVWarp = 9;          // V ring
 constexpr int kMmaWarp = 11;
 constexpr int kSoftmaxThreads = 256;       // two warpgroups
 constexpr int kBarSoftmax = 1;             // named barrier among the softmax warps
@@ -94,6 +95,47 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
       "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      KV_W32(v)
+      : "memory");
+}
+#define KV_R16(p) "=r"(p[0]), "=r"(p[1]), "=r"(p[2]), "=r"(p[3]), "=r"(p[4]), "=r"(p[5]), "=r"(p[6]), "=r"(p[7]), \
+    "=r"(p[8]), "=r"(p[9]), "=r"(p[10]), "=r"(p[11]), "=r"(p[12]), "=r"(p[13]), "=r"(p[14]), "=r"(p[15])
+
+// 16 lanes (from the address's lane) x 16 columns: threads 0..15 read columns
+// [col, col + 16) of lanes 0..15, threads 16..31 columns [col + 16, col + 32)
+// of the same lanes.
+__device__ __forceinline__ void tmem_ld16x2_16(uint32_t taddr, uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15}, [%16], 16;"
+      : KV_R16(v)
+      : "r"(taddr)
+      : "memory");
+}
+// 16 lanes x 32 columns: threads 0..15 columns [col, col + 32), threads 16..31
+// columns [col + 32, col + 64) of the same lanes.
+__device__ __forceinline__ void tmem_ld16x2_32_s32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32], 32;"
+      : KV_R32(v)
+      : "r"(taddr)
+      : "memory");
+}
+// 16 lanes x 32 columns: threads 0..15 columns [col, col + 32), threads 16..31
+// columns [col + 64, col + 96) of the same lanes.
+__device__ __forceinline__ void tmem_ld16x2_32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32], 64;"
+      : KV_R32(v)
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st16x2_32(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x32bx2.x32.b32 [%0], 64, {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
+      "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
       KV_W32(v)
       : "memory");
 }
@@ -193,10 +235,10 @@ __device__ Smem carve(uint8_t* raw, int C) {
 
 struct PendingPV {
   int tile, piece;
-  bool first;
+  bool first;  // first P.V into O_(tile % 2) of this piece: overwrite instead of accumulate
 };
 
-// O_w += P[:, 32w..32w+32) V[32w..32w+32, :] for both warpgroups w.
+// O_w += P V for tile t, w = t % 2 (the warpgroup that wrote P).
 __device__ __forceinline__ bool pv_ready(const Smem& sm, const PendingPV& pv) {
   if (!mbar_test_wait(smem_addr(&sm.vfull[pv.tile % kNV]), (pv.tile / kNV) & 1)) return false;
   if (!mbar_test_wait(smem_addr(&sm.pfull[pv.tile % kNP]), (pv.tile / kNP) & 1)) return false;
@@ -209,16 +251,14 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, const Pe
   constexpr uint32_t idesc = idesc_bf16(128, 128, true);
   const uint32_t pbase = smem_addr(sm.pbuf + b * kPBufBytes);
   const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(pv.tile % kNV) * kKVBytes);
+  const uint32_t o = tmem + kTmemO + 128 * (pv.tile & 1);
 #pragma unroll
-  for (int w = 0; w < 2; ++w)
-#pragma unroll
-    for (int kk = 0; kk < 2; ++kk) {
-      const int k16 = 2 * w + kk;  // 16-key step of the tile
-      const uint64_t a = smem_desc_sw128(pbase + k16 * 32, 16, 1024);
-      // V tile is MN-major: 64-dim halves 8 KB apart (leading), 8-key groups 1 KB apart (stride).
-      const uint64_t bd = smem_desc_sw128(vbase + k16 * 2048, kHalfBytes, 1024);
-      tc_mma(tmem + kTmemO + 128 * w, a, bd, idesc, (pv.first && kk == 0) ? 0u : 1u);
-    }
+  for (int k16 = 0; k16 < kTileKeys / 16; ++k16) {  // 16-key steps of the tile
+    const uint64_t a = smem_desc_sw128(pbase + k16 * 32, 16, 1024);
+    // V tile is MN-major: 64-dim halves 8 KB apart (leading), 8-key groups 1 KB apart (stride).
+    const uint64_t bd = smem_desc_sw128(vbase + k16 * 2048, kHalfBytes, 1024);
+    tc_mma(o, a, bd, idesc, (pv.first && k16 == 0) ? 0u : 1u);
+  }
   tc_commit(smem_addr(&sm.vempty[pv.tile % kNV]));
   tc_commit(smem_addr(&sm.pvdone[b]));
 }
@@ -229,7 +269,7 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, const Pe
 __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                         Cursor cu) {
   constexpr uint32_t idesc = idesc_bf16(128, 64, false);
-  int next_qk = 0, next_pv = 0, piece = 0, cur_piece = 0;
+  int next_qk = 0, next_pv = 0, piece = 0, cur_piece = 0, piece_t0 = 0;
   bool q_ready = false;  // the q block of the tile at the cursor is resident
   PendingPV pend[kNS];
   uint64_t idle_since = 0;
@@ -242,6 +282,7 @@ __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, con
       if ((!ti.first || q_ready) && mbar_test_wait(smem_addr(&sm.kfull[next_qk % kNK]), (next_qk / kNK) & 1)) {
         if (ti.first) {
           cur_piece = piece++;
+          piece_t0 = next_qk;
           sm.misc[4] = piece;
           q_ready = false;
         }
@@ -258,7 +299,7 @@ __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, con
         tc_commit(smem_addr(&sm.sfull[next_qk % kNS]));
         tc_commit(smem_addr(&sm.kempty[next_qk % kNK]));
         if (ti.last) tc_commit(smem_addr(sm.qempty));
-        pend[next_qk % kNS] = PendingPV{next_qk, cur_piece, ti.first};
+        pend[next_qk % kNS] = PendingPV{next_qk, cur_piece, next_qk - piece_t0 < 2};
         ++next_qk;
         cursor_next(cu, p, sm.len);
         progressed = true;
@@ -291,12 +332,30 @@ __device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, con
 
 // ------------------------------------------------------------ softmax + epilogue
 
+// Tile ownership: warpgroup w takes the tiles t with t % 2 == w (all 64 keys)
+// with its own running max/sum and its own accumulator O_w in TMEM, so two
+// tiles' softmax chains (S load, exponentials, P store) overlap; the two
+// states are merged by log-sum-exp at the end of each piece.
+// Row layout.  Dense units (more than 64 rows): thread = TMEM lane = stacked
+// row 32 quarter + lane, holding all 64 S columns.  Spread units (at most 64
+// rows): lanes 0..15 of each 32-lane quarter hold stacked rows 16 quarter +
+// 0..15, so every SM sub-partition's softmax warps get rows; two threads share
+// a lane (row), each with 32 of the 64 columns, and agree on the row max by
+// one shuffle.
+template <bool kSpread>
 __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                             Cursor cu) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int quarter = warp & 3;                 // TMEM lanes this warp may access
-  const int wg = warp >> 2;                     // warpgroup: key columns [32 wg, 32 wg + 32)
-  const int r = quarter * 32 + lane;            // accumulator row of this thread
+  const int wg = warp >> 2;                     // warpgroup: owns tiles t with t % 2 == wg
+  const int wtid = threadIdx.x & 127;           // thread within the warpgroup
+  const int half = kSpread ? lane >> 4 : 0;     // spread: which 32 of the 64 columns
+  const int tl = quarter * 32 + (kSpread ? (lane & 15) : lane);  // TMEM lane = row of the P buffer
+  const int r = kSpread ? quarter * 16 + (lane & 15) : tl;       // stacked row of the unit
+  constexpr int kCols = kSpread ? 32 : 64;      // S columns per thread
+  constexpr int kOChunks = kSpread ? 2 : 4;     // 32-column O chunks per thread
+  const int col0 = kCols * half;                // first S column of this thread
+  const int warp_row0 = kSpread ? quarter * 16 : quarter * 32;
   const int tid = threadIdx.x;                  // 0..255 among the softmax threads
   const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
   const uint32_t my_o = trow + kTmemO + 128 * wg;
@@ -305,16 +364,24 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
   const float qscale = p.qscale;
   const bool tree = p.tree != 0;
   const int nq = p.Nq, n_nodes = p.N;
-  float m_run = -INFINITY, l_run = 0.f;
+  // Row bookkeeping of the current unit, recomputed when the unit changes.
+  int unit_c = -1, unit_hr = -1, h = 0, rr = 0, nl = 0;
+  bool valid = false, warp_live = false;
+  float m_run = -INFINITY, l_run = 0.f;  // l_run: this thread's columns only (spread)
   int t = 0, anc_seq = -1;
   for (; cu.t < cu.t_end; cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
-    const int h = cu.hr / p.row_blocks, rb = cu.hr - h * p.row_blocks;
-    const int rows_blk = min(p.rows_per_unit, p.rows_total - rb * p.rows_per_unit);
-    const bool valid = r < rows_blk;
-    const bool warp_live = quarter * 32 < rows_blk;
-    const int rr = rb * p.rows_per_unit + r;
-    const int nl = valid ? rr / p.G : 0;
+    if (cu.c != unit_c || cu.hr != unit_hr) {
+      unit_c = cu.c;
+      unit_hr = cu.hr;
+      h = cu.hr / p.row_blocks;
+      const int rb = cu.hr - h * p.row_blocks;
+      const int rows_blk = min(p.rows_per_unit, p.rows_total - rb * p.rows_per_unit);
+      valid = r < rows_blk;
+      warp_live = warp_row0 < rows_blk;
+      rr = rb * p.rows_per_unit + r;
+      nl = valid ? rr / p.G : 0;
+    }
     if (ti.first) {
       m_run = -INFINITY;
       l_run = 0.f;
@@ -326,117 +393,131 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         anc_seq = seq;
       }
     }
-    const int sbuf = t % kNS, b = t % kNP;
     bool live = !*pipe.abort;
-    if (live && !mbar_wait(smem_addr(&sm.sfull[sbuf]), (t / kNS) & 1, p.err)) {
-      *pipe.abort = 1;
-      live = false;
-    }
-    live = __all_sync(0xffffffffu, live);
-    tc_fence_after();
-    float pr[32];
-    if (live && warp_live) {
-      uint32_t sv[32];
-      tmem_ld32(trow + sbuf * kTileKeys + 32 * wg, sv);
-      tmem_wait_ld();
-      // Visible keys of this row among the warpgroup's 32 columns (bit j = column 32 wg + j).
-      uint32_t vis = 0;
-      if (valid) {
-        uint64_t v64 = ti.nkeys >= 64 ? ~0ull : ((1ull << ti.nkeys) - 1ull);
-        if (ti.draft) {
-          uint64_t dm;
-          if (tree) {
-            dm = sm.anc[min(nl, nq - 1)] >> ti.key0;  // tree drafts have N <= 64, so key0 == 0
-          } else {
-            const int last = n_nodes - nq + nl - ti.key0;  // chain: slots key0 .. node are visible
-            dm = last >= 63 ? ~0ull : (last < 0 ? 0ull : ((2ull << last) - 1ull));
+    if ((t & 1) == wg) {
+      const int sbuf = t % kNS, b = t % kNP;
+      if (live && !mbar_wait(smem_addr(&sm.sfull[sbuf]), (t / kNS) & 1, p.err)) {
+        *pipe.abort = 1;
+        live = false;
+      }
+      live = __all_sync(0xffffffffu, live);
+      tc_fence_after();
+      float pr[kCols];
+      if (live && warp_live) {
+        uint32_t sv[kCols];
+        if constexpr (kSpread) {
+          tmem_ld16x2_32_s32(trow + sbuf * kTileKeys, sv);
+        } else {
+          tmem_ld32(trow + sbuf * kTileKeys, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+          tmem_ld32(trow + sbuf * kTileKeys + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+        }
+        tmem_wait_ld();
+        // Visible keys of this row (bit j = key key0 + j).
+        uint64_t v64 = 0;
+        if (valid) {
+          v64 = ti.nkeys >= 64 ? ~0ull : ((1ull << ti.nkeys) - 1ull);
+          if (ti.draft) {
+            uint64_t dm;
+            if (tree) {
+              dm = sm.anc[min(nl, nq - 1)] >> ti.key0;  // tree drafts have N <= 64, so key0 == 0
+            } else {
+              const int last = n_nodes - nq + nl - ti.key0;  // chain: slots key0 .. node are visible
+              dm = last >= 63 ? ~0ull : (last < 0 ? 0ull : ((2ull << last) - 1ull));
+            }
+            v64 &= dm;
           }
-          v64 &= dm;
         }
-        vis = static_cast<uint32_t>(v64 >> (32 * wg));
-      }
-      float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        const uint64_t vis = v64 >> col0;  // bit j = column col0 + j
+        float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * qscale : -INFINITY;
-        mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
-      }
-      const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
-      // Lazy rescale: move this row's reference max only when it grows by > 2^8.
-      const bool grow = valid && (m_run == -INFINITY ? mx != -INFINITY : mx > m_run + kRescaleThreshold);
-      const bool rescale_o = grow && m_run != -INFINITY;
-      if (__any_sync(0xffffffffu, rescale_o)) {
-        // O_wg must hold P.V of the previous tile before it is scaled.
-        if (!mbar_wait(smem_addr(&sm.pvdone[(t - 1) % kNP]), ((t - 1) / kNP) & 1, p.err)) *pipe.abort = 1;
-        tc_fence_after();
-        const float alpha = rescale_o ? ex2(m_run - mx) : 1.f;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          uint32_t o[32];
-          tmem_ld32(my_o + 32 * c, o);
-          tmem_wait_ld();
-#pragma unroll
-          for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha);
-          tmem_st32(my_o + 32 * c, o);
+        for (int j = 0; j < kCols; ++j) {
+          pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * qscale : -INFINITY;
+          mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
         }
-        tmem_wait_st();
-        l_run *= alpha;
-      }
-      if (grow) m_run = mx;
-      const float m_use = m_run == -INFINITY ? 0.f : m_run;
-      float ps4[4] = {0.f, 0.f, 0.f, 0.f};
+        float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+        if constexpr (kSpread) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+        // Lazy rescale: move this row's reference max only when it grows by > 2^8.
+        const bool grow = valid && (m_run == -INFINITY ? mx != -INFINITY : mx > m_run + kRescaleThreshold);
+        const bool rescale_o = grow && m_run != -INFINITY;
+        if (__any_sync(0xffffffffu, rescale_o)) {
+          // O_wg must hold P.V of this warpgroup's previous tile (t - 2) before it is scaled.
+          if (!mbar_wait(smem_addr(&sm.pvdone[(t - 2) % kNP]), ((t - 2) / kNP) & 1, p.err)) *pipe.abort = 1;
+          tc_fence_after();
+          const float alpha = rescale_o ? ex2(m_run - mx) : 1.f;
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        pr[j] = ex2(pr[j] - m_use);
-        ps4[j & 3] += pr[j];
-      }
-      l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
-    }
-    // The P buffer is free once P.V of tile t - kNP has completed.
-    if (live && t >= kNP && !mbar_wait(smem_addr(&sm.pvdone[b]), ((t - kNP) / kNP) & 1, p.err)) *pipe.abort = 1;
-    if (live && valid) {
-      uint8_t* prow = sm.pbuf + b * kPBufBytes + r * 128;
+          for (int c = 0; c < kOChunks; ++c) {
+            uint32_t o[32];
+            if constexpr (kSpread) tmem_ld16x2_32(my_o + 32 * c, o);
+            else tmem_ld32(my_o + 32 * c, o);
+            tmem_wait_ld();
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int chunk = 4 * wg + c;  // 16-byte chunk = 8 keys
-        uint4 w;
-        w.x = pack_bf16x2(pr[8 * c + 0], pr[8 * c + 1]);
-        w.y = pack_bf16x2(pr[8 * c + 2], pr[8 * c + 3]);
-        w.z = pack_bf16x2(pr[8 * c + 4], pr[8 * c + 5]);
-        w.w = pack_bf16x2(pr[8 * c + 6], pr[8 * c + 7]);
-        *reinterpret_cast<uint4*>(prow + ((chunk ^ (r & 7)) << 4)) = w;
+            for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha);
+            if constexpr (kSpread) tmem_st16x2_32(my_o + 32 * c, o);
+            else tmem_st32(my_o + 32 * c, o);
+          }
+          tmem_wait_st();
+          l_run *= alpha;
+        }
+        if (grow) m_run = mx;
+        const float m_use = m_run == -INFINITY ? 0.f : m_run;
+        float ps4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int j = 0; j < kCols; ++j) {
+          pr[j] = ex2(pr[j] - m_use);
+          ps4[j & 3] += pr[j];
+        }
+        l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
       }
-    }
-    if (live && ti.nkeys < kTileKeys) {
-      // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.
-      if (!mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err)) *pipe.abort = 1;
-      uint8_t* vptr = sm.vring + static_cast<size_t>(t % kNV) * kKVBytes;
-      const int nz = (kTileKeys - ti.nkeys) * 16;
-      for (int i = tid; i < nz; i += kSoftmaxThreads) {
-        const int key = ti.nkeys + (i >> 4), ch = i & 15;
-        *reinterpret_cast<uint4*>(vptr + tile_off(key, ch)) = make_uint4(0, 0, 0, 0);
+      // The P buffer is free once P.V of tile t - kNP has completed.
+      if (live && t >= kNP && !mbar_wait(smem_addr(&sm.pvdone[b]), ((t - kNP) / kNP) & 1, p.err)) *pipe.abort = 1;
+      if (live && valid) {
+        uint8_t* prow = sm.pbuf + b * kPBufBytes + tl * 128;
+#pragma unroll
+        for (int c = 0; c < kCols / 8; ++c) {
+          const int chunk = (col0 >> 3) + c;  // 16-byte chunk = 8 keys
+          uint4 w;
+          w.x = pack_bf16x2(pr[8 * c + 0], pr[8 * c + 1]);
+          w.y = pack_bf16x2(pr[8 * c + 2], pr[8 * c + 3]);
+          w.z = pack_bf16x2(pr[8 * c + 4], pr[8 * c + 5]);
+          w.w = pack_bf16x2(pr[8 * c + 6], pr[8 * c + 7]);
+          *reinterpret_cast<uint4*>(prow + ((chunk ^ (tl & 7)) << 4)) = w;
+        }
       }
+      if (live && ti.nkeys < kTileKeys) {
+        // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.
+        if (!mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err)) *pipe.abort = 1;
+        uint8_t* vptr = sm.vring + static_cast<size_t>(t % kNV) * kKVBytes;
+        const int nz = (kTileKeys - ti.nkeys) * 16;
+        for (int i = wtid; i < nz; i += kSoftmaxThreads / 2) {
+          const int key = ti.nkeys + (i >> 4), ch = i & 15;
+          *reinterpret_cast<uint4*>(vptr + tile_off(key, ch)) = make_uint4(0, 0, 0, 0);
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(smem_addr(&sm.pfull[b]));
     }
-    fence_proxy_async_smem();
-    tc_fence_before();
-    mbar_arrive(smem_addr(&sm.pfull[b]));
     if (ti.last) {
+      const int b = t % kNP;
       bool ok = live && mbar_wait(smem_addr(&sm.pvdone[b]), (t / kNP) & 1, p.err);
       ok = __all_sync(0xffffffffu, ok);
       tc_fence_after();
+      float l_row = l_run;
+      if constexpr (kSpread) l_row += __shfl_xor_sync(0xffffffffu, l_run, 16);
       // Merge the two warpgroups' states: warpgroup 1 publishes (max, sum), warpgroup 0 writes the row.
       if (wg == 1) {
-        sm.comb[2 * r] = m_run;
-        sm.comb[2 * r + 1] = l_run;
+        sm.comb[2 * tl] = m_run;
+        sm.comb[2 * tl + 1] = l_row;
       }
       named_barrier_sync(kBarSoftmax, kSoftmaxThreads);
       if (wg == 0 && ok && warp_live) {
-        const float m1 = sm.comb[2 * r], l1 = sm.comb[2 * r + 1];
+        const float m1 = sm.comb[2 * tl], l1 = sm.comb[2 * tl + 1];
         const float M = fmaxf(m_run, m1);
         const float w0 = m_run == -INFINITY ? 0.f : ex2(m_run - M);
         const float w1 = m1 == -INFINITY ? 0.f : ex2(m1 - M);
-        const float L = w0 * l_run + w1 * l1;
+        const float L = w0 * l_row + w1 * l1;
         const float inv = L > 0.f ? 1.f / L : 0.f;
+        // A warpgroup that owned no tile of this piece left O_w untouched: its weight is 0 and O_w is skipped.
         const float a0 = w0 * inv, a1 = w1 * inv;
         const float lse2 = L > 0.f ? M + __log2f(L) : -INFINITY;
         const bool whole = cu.lt == cu.ut - 1 && (cu.t - cu.t_begin) >= cu.lt;
@@ -447,17 +528,24 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
           orow = (static_cast<size_t>(cu.c) * p.Nq + nl) * p.hq + h * p.G + g;
         }
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < kOChunks; ++c) {
           uint32_t o0[32], o1[32];
-          tmem_ld32(trow + kTmemO + 32 * c, o0);
-          tmem_ld32(trow + kTmemO + 128 + 32 * c, o1);
+          if constexpr (kSpread) {
+            tmem_ld16x2_32(trow + kTmemO + 32 * c, o0);
+            tmem_ld16x2_32(trow + kTmemO + 128 + 32 * c, o1);
+          } else {
+            tmem_ld32(trow + kTmemO + 32 * c, o0);
+            tmem_ld32(trow + kTmemO + 128 + 32 * c, o1);
+          }
           tmem_wait_ld();
+          const int d0 = kSpread ? 64 * half + 32 * c : 32 * c;  // first output dim of this chunk
           float v[32];
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = a0 * __uint_as_float(o0[j]) + a1 * __uint_as_float(o1[j]);
+          for (int j = 0; j < 32; ++j)
+            v[j] = (a0 != 0.f ? a0 * __uint_as_float(o0[j]) : 0.f) + (a1 != 0.f ? a1 * __uint_as_float(o1[j]) : 0.f);
           if (valid) {
             if (whole) {
-              uint4* dst = reinterpret_cast<uint4*>(p.out + orow * kHeadDim + 32 * c);
+              uint4* dst = reinterpret_cast<uint4*>(p.out + orow * kHeadDim + d0);
 #pragma unroll
               for (int k = 0; k < 4; ++k) {
                 uint4 w;
@@ -469,13 +557,13 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
               }
             } else {
               float4* dst = reinterpret_cast<float4*>(
-                  p.ws_o + (static_cast<size_t>(slot) * p.rows_per_unit + r) * kHeadDim + 32 * c);
+                  p.ws_o + (static_cast<size_t>(slot) * p.rows_per_unit + r) * kHeadDim + d0);
 #pragma unroll
               for (int k = 0; k < 8; ++k) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
             }
           }
         }
-        if (valid) {
+        if (valid && half == 0) {
           if (whole) p.lse[orow] = lse2 * 0.69314718055994531f;
           else p.ws_lse[static_cast<size_t>(slot) * p.rows_per_unit + r] = lse2;
         }
@@ -490,10 +578,15 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
 
 // ------------------------------------------------------------ TMA producer
 
-// Walks this CTA's tiles: one q block per piece (single buffer), the K tile
-// into the K ring and the V tile into the V ring, each box from its own lane.
+// Walks this CTA's tiles and loads one of the two rings, each box from its
+// own lane: role 0 loads the K ring and one q block per piece (single
+// buffer), role 1 the V ring.  Two producer warps keep twice the loads in
+// flight that one warp can (a warp's bulk-tensor issues stall while its
+// earlier ones are outstanding).  A spread unit's q block goes in boxes of 16
+// stacked rows, box k to TMEM lanes (= q buffer rows) 32 k .. 32 k + 15.
+template <bool kSpread>
 __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const TensorMaps& maps, const Smem& sm,
-                                                const Pipe& pipe, Cursor cu, int nq_box) {
+                                                const Pipe& pipe, Cursor cu, int nq_box, int kv) {
   const int lane = threadIdx.x & 31;
   const uint64_t policy = l2_policy_evict_first();
   PageWindow win;
@@ -528,39 +621,46 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
     else y = (cu.c * p.hkv + h) * p.l_cap + key0;
     const uint32_t tx = nbox * br * 128 * 2;  // bytes of one K (or V) tile's boxes
     int ok = 1;
-    if (cu.t == cu.t_begin || cu.lt == 0) {  // first tile of a piece: the unit's q block
+    if (kv == 0 && (cu.t == cu.t_begin || cu.lt == 0)) {  // first tile of a piece: the unit's q block
       if (lane == 0) {
         const uint32_t qbar = smem_addr(sm.qfull);
         ok = mbar_wait(smem_addr(sm.qempty), (piece & 1) ^ 1u, p.err) && !*pipe.abort;
         if (ok) {
           const int rb = cu.hr - h * p.row_blocks;
           const uint32_t dst = smem_addr(sm.qbuf);
-          mbar_arrive_expect_tx(qbar, 2 * rows_q * 128);
-          tma_load_4d(dst, &maps.q, 0, h * p.G, rb * nq_box, cu.c, qbar);
-          tma_load_4d(dst + kQRows * 128, &maps.q, 64, h * p.G, rb * nq_box, cu.c, qbar);
+          const QBox qb = q_box(p.G, nq_box, kSpread);
+          const int box_rows = qb.heads * qb.nodes;
+          const int nqb = kSpread ? (rows_q + box_rows - 1) / box_rows : 1;
+          mbar_arrive_expect_tx(qbar, 2 * nqb * box_rows * 128);
+          for (int k = 0; k < nqb; ++k) {
+            const int s0 = k * box_rows;  // first stacked row of the box
+            const uint32_t d = dst + k * 32 * 128;
+            tma_load_4d(d, &maps.q, 0, h * p.G + s0 % p.G, rb * nq_box + s0 / p.G, cu.c, qbar);
+            tma_load_4d(d + kQRows * 128, &maps.q, 64, h * p.G + s0 % p.G, rb * nq_box + s0 / p.G, cu.c, qbar);
+          }
           sm.misc[3] = piece + 1;
         }
       }
       ++piece;
     }
-#pragma unroll
-    for (int kv = 0; kv < 2; ++kv) {
+    {
       const int slot = kv ? t % kNV : t % kNK;
       const int round = kv ? t / kNV : t / kNK;
       uint64_t* fullb = kv ? &sm.vfull[slot] : &sm.kfull[slot];
       uint64_t* emptyb = kv ? &sm.vempty[slot] : &sm.kempty[slot];
       if (lane == 0 && ok) ok = mbar_wait(smem_addr(emptyb), (round & 1) ^ 1u, p.err) && !*pipe.abort;
       ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) break;
-      const uint32_t full_bar = smem_addr(fullb);
-      if (lane == 0) mbar_arrive_expect_tx(full_bar, tx);
-      if (i < nbox) {
-        const uint32_t dst = smem_addr((kv ? sm.vring : sm.kring) + static_cast<size_t>(slot) * kKVBytes) +
-                             hf * kHalfBytes + i * br * 128;
-        const CUtensorMap* map = draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
-        tma_load_2d(dst, map, hf * 64, y, full_bar, policy);
+      if (ok) {
+        const uint32_t full_bar = smem_addr(fullb);
+        if (lane == 0) mbar_arrive_expect_tx(full_bar, tx);
+        if (i < nbox) {
+          const uint32_t dst = smem_addr((kv ? sm.vring : sm.kring) + static_cast<size_t>(slot) * kKVBytes) +
+                               hf * kHalfBytes + i * br * 128;
+          const CUtensorMap* map = draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
+          tma_load_2d(dst, map, hf * 64, y, full_bar, policy);
+        }
+        if (lane == 0) sm.misc[kv ? 5 : 1] = t + 1;
       }
-      if (lane == 0) sm.misc[kv ? 5 : 1] = t + 1;
     }
     if (!ok) {
       if (lane == 0) *pipe.abort = 1;
@@ -571,6 +671,7 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
   }
 }
 
+template <bool kSpread>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ TensorMaps maps, int nq_box) {
   extern __shared__ uint8_t smem_raw[];
@@ -589,7 +690,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(smem_addr(sm.qempty), 1);
     for (int b = 0; b < kNS; ++b) mbar_init(smem_addr(&sm.sfull[b]), 1);
     for (int b = 0; b < kNP; ++b) {
-      mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads);
+      mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads / 2);
       mbar_init(smem_addr(&sm.pvdone[b]), 1);
     }
     mbar_init(smem_addr(sm.ofree), kSoftmaxThreads);
@@ -612,8 +713,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *sm.tmem_base;
   const Cursor cu = cursor_begin(p, sm.len, sm.base);
   Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
-  if (warp == kProducerWarp) {
-    run_producer_tc(p, maps, sm, pipe, cu, nq_box);
+  if (warp == kProducerWarp || warp == kProducerVWarp) {
+    run_producer_tc<kSpread>(p, maps, sm, pipe, cu, nq_box, warp == kProducerVWarp ? 1 : 0);
   } else if (warp == kMmaWarp) {
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
       run_mma(p, sm, pipe, tmem, cu);
@@ -622,7 +723,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else if (warp < 8) {
-    run_softmax(p, sm, pipe, tmem, cu);
+    run_softmax<kSpread>(p, sm, pipe, tmem, cu);
   }
   tc_fence_before();
   __syncthreads();
@@ -643,18 +744,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 cudaError_t attn_tc_occupancy(int C, int* ctas_per_sm) {
   const size_t smem = smem_bytes(C);
-  cudaError_t e =
-      cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, attn_tc_kernel, kThreads, smem);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, attn_tc_kernel<false>, kThreads, smem);
 }
 
-cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, cudaStream_t stream) {
+cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, cudaStream_t stream) {
   const size_t smem = smem_bytes(p.C);
-  cudaError_t e =
-      cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  auto* kernel = spread ? attn_tc_kernel<true> : attn_tc_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  attn_tc_kernel<<<p.num_ctas, kThreads, smem, stream>>>(p, maps, nq_box);
+  kernel<<<p.num_ctas, kThreads, smem, stream>>>(p, maps, nq_box);
   return cudaGetLastError();
 }
 

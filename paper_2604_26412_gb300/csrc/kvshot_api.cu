@@ -56,15 +56,15 @@ bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box
 enum class Kernel { kCudaCore, kMma, kTensorMemory };
 
 // 4-D view {128 dims, hq, Nq, C} of q [C, Nq, hq, 128]; a box is one 64-dim
-// half of the G heads of one KV group for nq_box draft nodes (rows node-major).
-bool encode_q(CUtensorMap* map, const void* q, int C, int Nq, int hq, int G, int nq_box) {
+// half of `heads` heads of one KV group for `nodes` draft nodes (rows node-major).
+bool encode_q(CUtensorMap* map, const void* q, int C, int Nq, int hq, QBox qb) {
   auto fn = encode_fn();
   if (fn == nullptr) return false;
   const cuuint64_t dims[4] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(hq),
                               static_cast<cuuint64_t>(Nq), static_cast<cuuint64_t>(C)};
   const cuuint64_t row = static_cast<cuuint64_t>(kHeadDim) * 2;
   const cuuint64_t strides[3] = {row, row * hq, row * hq * Nq};
-  const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(nq_box), 1};
+  const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(qb.heads), static_cast<cuuint32_t>(qb.nodes), 1};
   const cuuint32_t estr[4] = {1, 1, 1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(q), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -76,6 +76,7 @@ struct Plan {
   bool mma;
   int m_tiles;        // mma path
   int nq_box;         // tensor-memory path: draft nodes per 128-row block
+  bool spread;        // tensor-memory path: 16 rows per TMEM lane quarter
   int rows_per_unit;
   int row_blocks;
   int units;
@@ -156,12 +157,14 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   pl->mma = pl->kernel == Kernel::kMma;
   pl->m_tiles = 0;
   pl->nq_box = 0;
+  pl->spread = false;
   if (pl->kernel == Kernel::kMma) {
     pl->m_tiles = std::min(kMmaMaxTiles, std::max(1, (rows + 15) / 16));
     pl->rows_per_unit = 16 * pl->m_tiles;
   } else if (pl->kernel == Kernel::kTensorMemory) {
     pl->nq_box = std::max(1, std::min(d->n_query, 128 / G));
     pl->rows_per_unit = G * pl->nq_box;
+    pl->spread = pl->rows_per_unit <= kSpreadMaxRows;
   } else {
     pl->rows_per_unit = kCcRows;
   }
@@ -255,7 +258,8 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
       !encode_rows(&maps.dk, draft_k, drows, kDraftBoxRows) || !encode_rows(&maps.dv, draft_v, drows, kDraftBoxRows))
     return KVSHOT_ERR_CUDA;
   if (pl.kernel == Kernel::kTensorMemory) {
-    if (!encode_q(&maps.q, q, d->num_caches, d->n_query, d->hq, d->hq / d->hkv, pl.nq_box)) return KVSHOT_ERR_CUDA;
+    if (!encode_q(&maps.q, q, d->num_caches, d->n_query, d->hq, q_box(d->hq / d->hkv, pl.nq_box, pl.spread)))
+      return KVSHOT_ERR_CUDA;
   } else {
     maps.q = maps.tk;  // unused by the other kernels
   }
@@ -298,7 +302,7 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = pl.kernel == Kernel::kMma            ? launch_attn_mma(p, maps, pl.m_tiles, s)
-                  : pl.kernel == Kernel::kTensorMemory ? launch_attn_tc(p, maps, pl.nq_box, s)
+                  : pl.kernel == Kernel::kTensorMemory ? launch_attn_tc(p, maps, pl.nq_box, pl.spread, s)
                                                        : launch_attn_cc(p, maps, s);
   if (e != cudaSuccess) return KVSHOT_ERR_CUDA;
   e = launch_merge(p, s);

@@ -32,6 +32,20 @@ constexpr int kMaxTreeNodes = 64;
 constexpr int kDraftBoxRows = 8;                      // draft K/V are loaded 8 rows per TMA box
 constexpr int kCcRows = 4;                            // rows per unit of the CUDA-core kernel
 constexpr int kMmaMaxTiles = 4;                       // m16 tiles per unit of the tensor-core kernel
+constexpr int kSpreadMaxRows = 64;                    // tensor-memory kernel: units up to this many rows are spread
+
+// Query box of the tensor-memory kernel's 4-D q map {128, hq, Nq, C}: `heads`
+// heads of the KV group x `nodes` draft nodes.  Dense units load all G x nq_box
+// stacked rows as one box.  Spread units (<= 64 rows) put 16 stacked rows in
+// each 32-lane TMEM quarter, so a box holds at most 16 rows.
+struct QBox {
+  int heads, nodes;
+};
+__host__ __device__ inline QBox q_box(int G, int nq_box, bool spread) {
+  if (!spread) return QBox{G, nq_box};
+  if (G >= 16) return QBox{16, 1};
+  return QBox{G, nq_box < 16 / G ? nq_box : 16 / G};
+}
 
 // Everything a draft-attention kernel needs besides the tensor maps.
 struct AttnParams {
@@ -78,7 +92,7 @@ struct TensorMaps {
 // Kernel launchers (one per translation unit).  Return cudaSuccess or the launch error.
 cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, cudaStream_t stream);
 cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, cudaStream_t stream);
-cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, cudaStream_t stream);
+cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, cudaStream_t stream);
 cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream);
 cudaError_t launch_append(const AppendParams& a, cudaStream_t stream);
 

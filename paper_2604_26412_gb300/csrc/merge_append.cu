@@ -12,55 +12,93 @@ namespace {
 
 using namespace dev;
 
-constexpr int kMergeThreads = 128;
+constexpr int kMergeThreads = 256;
+constexpr int kMergeRows = kMergeThreads / 32;  // rows per CTA, one warp per row
 
-// One CTA per unit.  Workspace slot of the piece computed by CTA b is u + b.
+// Workspace slot of the piece computed by CTA b is u + b.  One warp per row
+// of a unit; lane k reads the lse of piece b0 + k, and every piece's partial
+// output (lane = 4 dims) is read in one batch of independent loads.
 __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_constant__ AttnParams p) {
-  const int u = blockIdx.x;
+  const int blocks_per_unit = (p.rows_per_unit + kMergeRows - 1) / kMergeRows;
+  const int u = blockIdx.x / blocks_per_unit;
+  const int r = (blockIdx.x - u * blocks_per_unit) * kMergeRows + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
   const int HR = p.hkv * p.row_blocks;
   const int c = u / HR, hr = u - c * HR;
   const int h = hr / p.row_blocks, rb = hr - h * p.row_blocks;
+  const int rr = rb * p.rows_per_unit + r;
+  if (r >= p.rows_per_unit || rr >= p.rows_total) return;
   const int L = clamp_len(p, c);
   const int ut = (L + kTileKeys - 1) / kTileKeys + p.draft_tiles;
   const int gs = p.ws_meta[c] + hr * ut;
-  const int total = p.ws_meta[p.C];
-  const int tpc = tiles_per_cta(total, p.num_ctas);
+  const int tpc = tiles_per_cta(p.ws_meta[p.C], p.num_ctas);
   const int b0 = gs / tpc, b1 = (gs + ut - 1) / tpc;
   if (b0 == b1) return;  // the unit lived in one CTA, which wrote the output itself
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int r = warp; r < p.rows_per_unit; r += kMergeThreads / 32) {
-    const int rr = rb * p.rows_per_unit + r;
-    if (rr >= p.rows_total) break;
-    float M = -INFINITY;
-    for (int b = b0; b <= b1; ++b) M = fmaxf(M, p.ws_lse[static_cast<size_t>(u + b) * p.rows_per_unit + r]);
-    float Lsum = 0.f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (M != -INFINITY) {
-      for (int b = b0; b <= b1; ++b) {
-        const size_t row = static_cast<size_t>(u + b) * p.rows_per_unit + r;
-        const float ls = p.ws_lse[row];
-        if (ls == -INFINITY) continue;
-        const float w = exp2f(ls - M);
+  const int np = b1 - b0 + 1;
+  // Pass 1: the largest piece lse.
+  float M = -INFINITY;
+  for (int k = lane; k < np; k += 32)
+    M = fmaxf(M, p.ws_lse[static_cast<size_t>(u + b0 + k) * p.rows_per_unit + r]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  // Pass 2: weights e^(lse_s - M) and the weighted partial outputs.
+  float Lsum = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (M != -INFINITY) {
+    for (int k0 = 0; k0 < np; k0 += 32) {
+      const int k = k0 + lane;
+      float wl = 0.f;
+      if (k < np) {
+        const float ls = p.ws_lse[static_cast<size_t>(u + b0 + k) * p.rows_per_unit + r];
+        wl = ls == -INFINITY ? 0.f : exp2f(ls - M);
+      }
+      const int n = min(32, np - k0);
+      for (int j = 0; j < n; ++j) {
+        const float w = __shfl_sync(0xffffffffu, wl, j);
         Lsum += w;
-        const float4 v = *reinterpret_cast<const float4*>(p.ws_o + row * kHeadDim + 4 * lane);
-        acc.x += w * v.x;
-        acc.y += w * v.y;
-        acc.z += w * v.z;
-        acc.w += w * v.w;
+        if (w != 0.f) {
+          const size_t row = static_cast<size_t>(u + b0 + k0 + j) * p.rows_per_unit + r;
+          const float4 v = *reinterpret_cast<const float4*>(p.ws_o + row * kHeadDim + 4 * lane);
+          acc.x += w * v.x;
+          acc.y += w * v.y;
+          acc.z += w * v.z;
+          acc.w += w * v.w;
+        }
       }
     }
-    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-    const int nl = rr / p.G, g = rr - nl * p.G;
-    const size_t orow = (static_cast<size_t>(c) * p.Nq + nl) * p.hq + h * p.G + g;
-    uint2 packed;
-    packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-    packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-    *reinterpret_cast<uint2*>(p.out + orow * kHeadDim + 4 * lane) = packed;
-    if (lane == 0) p.lse[orow] = Lsum > 0.f ? (M + log2f(Lsum)) * 0.69314718055994531f : -INFINITY;
   }
+  const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+  const int nl = rr / p.G, g = rr - nl * p.G;
+  const size_t orow = (static_cast<size_t>(c) * p.Nq + nl) * p.hq + h * p.G + g;
+  uint2 packed;
+  packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+  packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+  *reinterpret_cast<uint2*>(p.out + orow * kHeadDim + 4 * lane) = packed;
+  if (lane == 0) p.lse[orow] = Lsum > 0.f ? (M + log2f(Lsum)) * 0.69314718055994531f : -INFINITY;
 }
 
 constexpr int kAppendThreads = 256;
+
+// One rotated component of RoPE, x' = a * cos - b * sin (sgn = -1) or
+// y' = b * cos + a * sin (sgn = +1), rounded to bf16 as the fp64 evaluation
+// rounds.  The fp32 value r differs from the exact a c + sgn b s by at most
+// 2^-24 (|a| + 2 |b| + |r|) (cos/sin rounded to fp32, one product and one fma
+// rounded); when r lies farther than twice that from every bf16 rounding
+// midpoint both round alike, otherwise the component is recomputed in fp64.
+__device__ __forceinline__ __nv_bfloat16 rope_bf16(float a, float b, float c32, float s32, double c, double s,
+                                                   float sgn) {
+  const float r = fmaf(a, c32, sgn * (b * s32));
+  const uint32_t u = __float_as_uint(r);
+  const int e = static_cast<int>((u >> 23) & 0xFFu);
+  const float bound = 0x1p-23f * (fabsf(a) + 2.f * fabsf(b) + fabsf(r));
+  if (e >= 40) {
+    const float ulp = __uint_as_float(static_cast<uint32_t>(e - 23) << 23);  // 2^(e - 150), fp32 spacing at r
+    const float dist = fabsf(static_cast<float>(static_cast<int>(u & 0xFFFFu) - 0x8000)) * ulp;
+    if (dist > bound) return __float2bfloat16_rn(r);
+  }
+  const double da = a, db = b;
+  return __double2bfloat16(sgn < 0.f ? da * c - db * s : da * c + db * s);
+}
 
 // One CTA per (cache, new node).  Work item = (head, 16-byte chunk j0 of the
 // first half): it rotates dims j0..j0+7 together with their partners +64.
@@ -99,10 +137,12 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(const __grid_con
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
         const int j = j0 + 2 * k + e;
-        const double x = e ? bf16_hi(wl[k]) : bf16_lo(wl[k]);
-        const double y = e ? bf16_hi(wh[k]) : bf16_lo(wh[k]);
-        rl[e] = __double2bfloat16(x * s_cos[j] - y * s_sin[j]);
-        rh[e] = __double2bfloat16(y * s_cos[j] + x * s_sin[j]);
+        const float x = e ? bf16_hi(wl[k]) : bf16_lo(wl[k]);
+        const float y = e ? bf16_hi(wh[k]) : bf16_lo(wh[k]);
+        const double cs = s_cos[j], sn = s_sin[j];
+        const float c32 = static_cast<float>(cs), s32 = static_cast<float>(sn);
+        rl[e] = rope_bf16(x, y, c32, s32, cs, sn, -1.f);
+        rh[e] = rope_bf16(y, x, c32, s32, cs, sn, 1.f);
       }
       ol[k] = static_cast<uint32_t>(__bfloat16_as_ushort(rl[0])) |
               (static_cast<uint32_t>(__bfloat16_as_ushort(rl[1])) << 16);
@@ -126,7 +166,8 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(const __grid_con
 
 cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream) {
   const int units = p.C * p.hkv * p.row_blocks;
-  merge_kernel<<<units, kMergeThreads, 0, stream>>>(p);
+  const int blocks = units * ((p.rows_per_unit + kMergeRows - 1) / kMergeRows);
+  merge_kernel<<<blocks, kMergeThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }
 

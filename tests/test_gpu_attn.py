@@ -1,9 +1,9 @@
 """GPU parity of kvshot_draft_attn against the CPU fp64 oracle (through the C ABI).
 
 Shapes span several 64-key tiles with ragged tails, empty prefixes, both cache
-layouts and several page sizes, chains and trees, GQA groups 1/4/8, the
-CUDA-core and tensor-core kernels, single-row and multi-row-block stacks, and
-persistent grids from 1 CTA up (which changes how units are split into
+layouts and several page sizes, chains and trees, GQA groups 1/4/8/16/32, the
+CUDA-core and tensor-core kernels (tensor-memory rows dense or spread),
+single-row and multi-row-block stacks, and persistent grids from 1 CTA up (which changes how units are split into
 pieces and merged).  Unused cache rows and draft slots hold NaN.
 """
 import math
@@ -67,6 +67,9 @@ CASES = [
     ((90, 91, 92), (2, 2, 2), False, True, 16, 64, 8, 2),         # G = 8, chain of 6 nodes, 16 rows
     ((1500,), tuple([1] * 40), False, True, 16, 32, 8, 1),        # long chain: two draft tiles? (N = 40)
     ((65,), tuple([1] * 70), False, False, 16, 4, 4, 2),          # chain with N = 70 > one draft tile
+    ((600, 129), (8, 12), True, True, 16, 32, 8, 20),             # 80 rows: dense TMEM rows, partial quarter
+    ((300,), (2, 2), True, False, 16, 32, 2, 3),                  # G = 16: 48 rows spread, boxes of one node
+    ((250, 70), (1, 1, 1), False, True, 16, 32, 1, 2),            # G = 32: 64 rows spread, boxes of 16 heads
 ]
 
 
