@@ -10,13 +10,14 @@
 // Warp roles: warps 0..7 are two softmax warpgroups; warp 10 loads K tiles
 // and the q block of each piece by TMA, warp 9 loads V tiles (a single warp
 // keeps too few bulk-tensor loads in flight to reach full HBM bandwidth);
-// warp 11 owns TMEM and one of its threads issues every MMA (warp 8 idles).
+// warp 11 owns TMEM and one of its threads issues every QK^T, one thread of
+// warp 8 every P.V.
 // Warpgroup w owns the tiles t with t % 2 == w: it turns S into P for all 64
 // keys with its own running max/sum and its own O accumulator O_w in TMEM, so
 // the two warpgroups' per-tile chains overlap; the states are merged by
-// log-sum-exp at the end of each piece.  S has four TMEM buffers; the MMA
-// thread issues QK^T as soon as a K tile and an S buffer are free and P.V as
-// soon as P is written, so QK^T runs ahead of the softmax.  O_w is rescaled in
+// log-sum-exp at the end of each piece.  S has four TMEM buffers; QK^T is
+// issued as soon as a K tile and an S buffer are free and P.V as soon as P is
+// written, so QK^T runs ahead of the softmax.  O_w is rescaled in
 // TMEM only when a row's running max grows by more than 2^8 (lazy rescale).
 // Rows of the 128-row MMA that hold no stacked row carry no output.
 #include "kvshot_attn_common.cuh"
@@ -34,7 +35,8 @@ constexpr int kNP = 3;                     // P buffers in shared memory
 constexpr int kThreads = 12 * 32;
 constexpr int kProducerWarp = 10;          // K ring and q blocks
 constexpr int kProducerVWarp = 9;          // V ring
-constexpr int kMmaWarp = 11;
+constexpr int kMmaWarp = 11;               // TMEM owner, QK^T issuer
+constexpr int kMmaPvWarp = 8;              // P.V issuer
 constexpr int kSoftmaxThreads = 256;       // two warpgroups
 constexpr int kBarSoftmax = 1;             // named barrier among the softmax warps
 constexpr int kPBufBytes = kQRows * 128;   // 128 rows x 64 keys bf16
@@ -168,17 +170,17 @@ struct Smem {
   uint8_t* vring;      // kNV x V tile
   uint8_t* qbuf;       // one q block
   uint8_t* pbuf;       // kNP x kPBufBytes
-  uint64_t* kfull;     // [kNK]  TMA -> MMA
-  uint64_t* kempty;    // [kNK]  QK^T completion -> TMA
+  uint64_t* kfull;     // [kNK]  TMA -> MMA (a K slot is free again once QK^T of its tile completed: sfull)
   uint64_t* vfull;     // [kNV]  TMA -> MMA, softmax
   uint64_t* vempty;    // [kNV]  P.V completion -> TMA
   uint64_t* qfull;     // [1]
   uint64_t* qempty;    // [1]
-  uint64_t* sfull;     // [kNS]  S buffer written (MMA completion)
+  uint64_t* sfull;     // [kNS]  S buffer written (QK^T completion)
+  uint64_t* sfree;     // [kNS]  S buffer read (the owning warpgroup's 128 threads)
   uint64_t* pfull;     // [kNP]  P buffer written and S consumed (256 softmax threads)
   uint64_t* pvdone;    // [kNP]  P.V of the tile using that buffer completed
   uint64_t* ofree;     // [1]  epilogue finished reading O
-  uint64_t* mmadone;   // [1]  every MMA completed
+  uint64_t* mmadone;   // [2]  every QK^T / every P.V completed
   uint64_t* anc;       // [64]
   int* par;            // [64]
   float* comb;         // [128][2] second warpgroup's (max, sum) per row at a piece end
@@ -190,7 +192,7 @@ struct Smem {
 
 __host__ __device__ inline size_t smem_bytes(int C) {
   size_t off = static_cast<size_t>(kNK + kNV) * kKVBytes + kQBufBytes + kNP * kPBufBytes;
-  off += sizeof(uint64_t) * (2 * kNK + 2 * kNV + 2 + kNS + 2 * kNP + 2);
+  off += sizeof(uint64_t) * (kNK + 2 * kNV + 2 + 2 * kNS + 2 * kNP + 3);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(float) * 2 * kQRows;
   off += sizeof(uint32_t) * 4 + sizeof(int) * 8;
@@ -211,17 +213,17 @@ __device__ Smem carve(uint8_t* raw, int C) {
   p += kNP * kPBufBytes;
   uint64_t* b = reinterpret_cast<uint64_t*>(p);
   s.kfull = b;
-  s.kempty = s.kfull + kNK;
-  s.vfull = s.kempty + kNK;
+  s.vfull = s.kfull + kNK;
   s.vempty = s.vfull + kNV;
   s.qfull = s.vempty + kNV;
   s.qempty = s.qfull + 1;
   s.sfull = s.qempty + 1;
-  s.pfull = s.sfull + kNS;
+  s.sfree = s.sfull + kNS;
+  s.pfull = s.sfree + kNS;
   s.pvdone = s.pfull + kNP;
   s.ofree = s.pvdone + kNP;
   s.mmadone = s.ofree + 1;
-  s.anc = s.mmadone + 1;
+  s.anc = s.mmadone + 2;
   s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
   s.comb = reinterpret_cast<float*>(s.par + kMaxTreeNodes);
   s.tmem_base = reinterpret_cast<uint32_t*>(s.comb + 2 * kQRows);
@@ -233,101 +235,82 @@ __device__ Smem carve(uint8_t* raw, int C) {
 
 // ------------------------------------------------------------ MMA issuer
 
-struct PendingPV {
-  int tile, piece;
-  bool first;  // first P.V into O_(tile % 2) of this piece: overwrite instead of accumulate
-};
+// Two threads issue the MMAs, one stream each, so that neither stream's
+// issue (which stalls while the tensor pipe is busy) delays the other:
+// QK^T in tile order from warp kMmaWarp, P.V in tile order from warp
+// kMmaPvWarp.  A tcgen05.commit tracks the MMAs of the thread that issues it.
 
-// O_w += P V for tile t, w = t % 2 (the warpgroup that wrote P).
-__device__ __forceinline__ bool pv_ready(const Smem& sm, const PendingPV& pv) {
-  if (!mbar_test_wait(smem_addr(&sm.vfull[pv.tile % kNV]), (pv.tile / kNV) & 1)) return false;
-  if (!mbar_test_wait(smem_addr(&sm.pfull[pv.tile % kNP]), (pv.tile / kNP) & 1)) return false;
-  return !(pv.first && pv.piece > 0) || mbar_test_wait(smem_addr(sm.ofree), (pv.piece - 1) & 1);
-}
-
-__device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, const PendingPV& pv) {
-  const int b = pv.tile % kNP;
-  tc_fence_after();
-  constexpr uint32_t idesc = idesc_bf16(128, 128, true);
-  const uint32_t pbase = smem_addr(sm.pbuf + b * kPBufBytes);
-  const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(pv.tile % kNV) * kKVBytes);
-  const uint32_t o = tmem + kTmemO + 128 * (pv.tile & 1);
-#pragma unroll
-  for (int k16 = 0; k16 < kTileKeys / 16; ++k16) {  // 16-key steps of the tile
-    const uint64_t a = smem_desc_sw128(pbase + k16 * 32, 16, 1024);
-    // V tile is MN-major: 64-dim halves 8 KB apart (leading), 8-key groups 1 KB apart (stride).
-    const uint64_t bd = smem_desc_sw128(vbase + k16 * 2048, kHalfBytes, 1024);
-    tc_mma(o, a, bd, idesc, (pv.first && k16 == 0) ? 0u : 1u);
-  }
-  tc_commit(smem_addr(&sm.vempty[pv.tile % kNV]));
-  tc_commit(smem_addr(&sm.pvdone[b]));
-}
-
-// Event-driven issue: each pass issues QK^T of the next tile if its K tile has
-// landed and an S buffer is free, and P.V of the oldest pending tile if its P
-// is written.  Nothing blocks, so QK^T runs ahead of the softmax.
-__device__ __forceinline__ void run_mma(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
-                                        Cursor cu) {
+// S = Q K^T of every tile.  Tile t needs its K tile, its S buffer read by the
+// softmax of tile t - kNS, and (first tile of a piece) the piece's q block.
+__device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
+                                           Cursor cu) {
   constexpr uint32_t idesc = idesc_bf16(128, 64, false);
-  int next_qk = 0, next_pv = 0, piece = 0, cur_piece = 0, piece_t0 = 0;
-  bool q_ready = false;  // the q block of the tile at the cursor is resident
-  PendingPV pend[kNS];
-  uint64_t idle_since = 0;
-  bool ok = true;
-  while (ok) {
-    bool progressed = false;
-    if (cu.t < cu.t_end && next_qk - next_pv < kNS) {
-      const TileInfo ti = tile_info(cu, p);
-      if (ti.first && !q_ready) q_ready = mbar_test_wait(smem_addr(sm.qfull), piece & 1);
-      if ((!ti.first || q_ready) && mbar_test_wait(smem_addr(&sm.kfull[next_qk % kNK]), (next_qk / kNK) & 1)) {
-        if (ti.first) {
-          cur_piece = piece++;
-          piece_t0 = next_qk;
-          sm.misc[4] = piece;
-          q_ready = false;
-        }
-        sm.misc[2] = next_qk + 1;
-        tc_fence_after();
-        const uint32_t qbase = smem_addr(sm.qbuf);
-        const uint32_t kbase = smem_addr(sm.kring + static_cast<size_t>(next_qk % kNK) * kKVBytes);
+  int piece = 0;
+  for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
+    const TileInfo ti = tile_info(cu, p);
+    bool ok = !*pipe.abort;
+    if (ok && ti.first) ok = mbar_wait(smem_addr(sm.qfull), piece & 1, p.err);
+    if (ok && t >= kNS) ok = mbar_wait(smem_addr(&sm.sfree[t % kNS]), ((t - kNS) / kNS) & 1, p.err);
+    if (ok) ok = mbar_wait(smem_addr(&sm.kfull[t % kNK]), (t / kNK) & 1, p.err);
+    if (!ok) {
+      *pipe.abort = 1;
+      break;
+    }
+    if (ti.first) sm.misc[4] = ++piece;
+    sm.misc[2] = t + 1;
+    tc_fence_after();
+    const uint32_t qbase = smem_addr(sm.qbuf);
+    const uint32_t kbase = smem_addr(sm.kring + static_cast<size_t>(t % kNK) * kKVBytes);
 #pragma unroll
-        for (int ks = 0; ks < kHeadDim / 16; ++ks) {
-          const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
-          const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * kHalfBytes + (ks & 3) * 32, 16, 1024);
-          tc_mma(tmem + (next_qk % kNS) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
-        }
-        tc_commit(smem_addr(&sm.sfull[next_qk % kNS]));
-        tc_commit(smem_addr(&sm.kempty[next_qk % kNK]));
-        if (ti.last) tc_commit(smem_addr(sm.qempty));
-        pend[next_qk % kNS] = PendingPV{next_qk, cur_piece, next_qk - piece_t0 < 2};
-        ++next_qk;
-        cursor_next(cu, p, sm.len);
-        progressed = true;
-      }
+    for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+      const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
+      const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * kHalfBytes + (ks & 3) * 32, 16, 1024);
+      tc_mma(tmem + (t % kNS) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
     }
-    if (next_pv < next_qk && pv_ready(sm, pend[next_pv % kNS])) {
-      issue_pv(sm, tmem, pend[next_pv % kNS]);
-      ++next_pv;
-      sm.misc[6] = next_pv;
-      progressed = true;
-    }
-    if (cu.t >= cu.t_end && next_pv == next_qk) break;
-    if (progressed) {
-      idle_since = 0;
-    } else if (*pipe.abort) {
-      ok = false;
-    } else {
-      const uint64_t now = global_timer_ns();
-      if (idle_since == 0) {
-        idle_since = now;
-      } else if (now - idle_since > kWaitLimitNs) {
-        set_error(p.err, KVSHOT_ERR_TIMEOUT);
-        ok = false;
-      }
-    }
+    tc_commit(smem_addr(&sm.sfull[t % kNS]));
+    if (ti.last) tc_commit(smem_addr(sm.qempty));
   }
-  if (!ok) *pipe.abort = 1;
-  tc_commit(smem_addr(sm.mmadone));
+  tc_commit(smem_addr(&sm.mmadone[0]));
+}
+
+// O_w += P V of every tile, w = t % 2 (the warpgroup that wrote P).  Tile t
+// needs its P and its V tile; the first P.V into O_w of a piece (which
+// overwrites O_w) needs the previous piece's epilogue to have read O.
+__device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
+                                           Cursor cu) {
+  constexpr uint32_t idesc = idesc_bf16(128, 128, true);
+  int piece = 0, piece_t0 = 0;
+  for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
+    const TileInfo ti = tile_info(cu, p);
+    if (ti.first) {
+      ++piece;
+      piece_t0 = t;
+    }
+    const bool first = t - piece_t0 < 2;
+    bool ok = !*pipe.abort;
+    if (ok && first && piece > 1) ok = mbar_wait(smem_addr(sm.ofree), (piece - 2) & 1, p.err);
+    if (ok) ok = mbar_wait(smem_addr(&sm.pfull[t % kNP]), (t / kNP) & 1, p.err);
+    if (ok) ok = mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err);
+    if (!ok) {
+      *pipe.abort = 1;
+      break;
+    }
+    sm.misc[6] = t + 1;
+    tc_fence_after();
+    const uint32_t pbase = smem_addr(sm.pbuf + (t % kNP) * kPBufBytes);
+    const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(t % kNV) * kKVBytes);
+    const uint32_t o = tmem + kTmemO + 128 * (t & 1);
+#pragma unroll
+    for (int k16 = 0; k16 < kTileKeys / 16; ++k16) {  // 16-key steps of the tile
+      const uint64_t a = smem_desc_sw128(pbase + k16 * 32, 16, 1024);
+      // V tile is MN-major: 64-dim halves 8 KB apart (leading), 8-key groups 1 KB apart (stride).
+      const uint64_t bd = smem_desc_sw128(vbase + k16 * 2048, kHalfBytes, 1024);
+      tc_mma(o, a, bd, idesc, (first && k16 == 0) ? 0u : 1u);
+    }
+    tc_commit(smem_addr(&sm.vempty[t % kNV]));
+    tc_commit(smem_addr(&sm.pvdone[t % kNP]));
+  }
+  tc_commit(smem_addr(&sm.mmadone[1]));
 }
 
 // ------------------------------------------------------------ softmax + epilogue
@@ -403,6 +386,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       live = __all_sync(0xffffffffu, live);
       tc_fence_after();
       float pr[kCols];
+      if (!(live && warp_live)) mbar_arrive(smem_addr(&sm.sfree[sbuf]));  // S is not read
       if (live && warp_live) {
         uint32_t sv[kCols];
         if constexpr (kSpread) {
@@ -412,6 +396,8 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
           tmem_ld32(trow + sbuf * kTileKeys + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
         }
         tmem_wait_ld();
+        tc_fence_before();
+        mbar_arrive(smem_addr(&sm.sfree[sbuf]));
         // Visible keys of this row (bit j = key key0 + j).
         uint64_t v64 = 0;
         if (valid) {
@@ -578,6 +564,60 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
 
 // ------------------------------------------------------------ TMA producer
 
+// Exact n / d for 0 <= n < 2^24 and 1 <= d <= 256 by a multiply-high with
+// m = ceil(2^32 / d): writing n = q d + r, the product overshoots n / d by
+// n (m d - 2^32) / (d 2^32) < 1 / d, which never carries r / d past 1.
+// Larger dividends (`small` false) take the hardware division.
+struct FastDiv {
+  uint32_t d, m;
+  bool exact;
+  __device__ __forceinline__ FastDiv(uint32_t dd, bool small)
+      : d(dd), m(dd > 1 ? 0xFFFFFFFFu / dd + 1u : 0u), exact(small && dd <= 256) {}
+  __device__ __forceinline__ int div(int n) const {
+    const uint32_t u = static_cast<uint32_t>(n);
+    return static_cast<int>(d == 1 ? u : (exact ? __umulhi(u, m) : u / d));
+  }
+};
+
+// TMA boxes of one K (or V) tile: `nbox` boxes of `br` rows in each 64-dim
+// half; lane (hf = lane & 1, i = lane >> 1) owns box i of half hf, whose first
+// row in the tile's tensor map (target or draft) is y.  h is the unit's KV
+// head, `pages` the cache's pages in use.  Warp-wide.
+struct TileBoxes {
+  bool draft;
+  int y, nbox, br;
+};
+
+__device__ __forceinline__ TileBoxes tile_boxes(const AttnParams& p, const Cursor& cu, PageWindow& win, int lane,
+                                                int h, int pages, const FastDiv& pdiv) {
+  TileBoxes tb;
+  tb.draft = cu.lt >= cu.pt;
+  const int key0 = (tb.draft ? cu.lt - cu.pt : cu.lt) * kTileKeys;
+  const int nkeys = min(kTileKeys, (tb.draft ? p.N : cu.L) - key0);
+  const int i = lane >> 1;
+  if (tb.draft) {
+    tb.br = kDraftBoxRows;
+    tb.nbox = (nkeys + kDraftBoxRows - 1) / kDraftBoxRows;
+    tb.y = (cu.c * p.hkv + h) * p.n_max + key0 + i * tb.br;
+  } else if (p.paged) {
+    // Pages of P <= 64 rows: one box per page (P divides the tile); larger
+    // pages: one 64-row box inside the page.
+    const int P = p.page_size;
+    tb.br = p.box_rows;
+    tb.nbox = tb.br < kTileKeys ? pdiv.div(nkeys + P - 1) : 1;
+    const int pg0 = pdiv.div(key0);
+    const int npg = tb.br < P ? 1 : tb.nbox;
+    win.cover(p, cu.c, pages, pg0, npg, lane);
+    const int pid = win.get(pg0 + (tb.br < P ? 0 : min(i, npg - 1)));
+    tb.y = (pid * p.hkv + h) * P + (tb.br < P ? key0 - pg0 * P : 0);
+  } else {
+    tb.br = kTileKeys;
+    tb.nbox = 1;
+    tb.y = (cu.c * p.hkv + h) * p.l_cap + key0;
+  }
+  return tb;
+}
+
 // Walks this CTA's tiles and loads one of the two rings, each box from its
 // own lane: role 0 loads the K ring and one q block per piece (single
 // buffer), role 1 the V ring.  Two producer warps keep twice the loads in
@@ -592,34 +632,20 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
   PageWindow win;
   int t = 0, piece = 0;
   const int rows_q = p.G * nq_box;
+  const bool small = p.len_bound < (1 << 24) - 2 * kTileKeys;
+  const FastDiv pdiv(p.paged ? p.page_size : 1, small), rbdiv(p.row_blocks, true);
+  int unit_c = -1, unit_hr = -1, h = 0, pages = 0;  // the current unit's KV head and its cache's pages
   while (cu.t < cu.t_end) {
-    const int h = cu.hr / p.row_blocks;
-    const bool draft = cu.lt >= cu.pt;
-    const int key0 = (draft ? cu.lt - cu.pt : cu.lt) * kTileKeys;
-    const int nkeys = min(kTileKeys, (draft ? p.N : cu.L) - key0);
-    int pid = 0;  // page id of this lane's box
-    int nbox, br;
-    if (draft) {
-      br = kDraftBoxRows;
-      nbox = (nkeys + br - 1) / br;
-    } else if (p.paged) {
-      br = p.box_rows;
-      nbox = (nkeys + br - 1) / br;
-      const int pg0 = key0 / p.page_size;
-      const int npg = br < p.page_size ? 1 : nbox;
-      win.cover(p, cu.c, (cu.L + p.page_size - 1) / p.page_size, pg0, npg, lane);
-      const int i = min(lane >> 1, npg - 1);
-      pid = win.get(pg0 + (br < p.page_size ? 0 : i));
-    } else {
-      br = kTileKeys;
-      nbox = 1;
+    if (cu.c != unit_c || cu.hr != unit_hr) {
+      unit_c = cu.c;
+      unit_hr = cu.hr;
+      h = rbdiv.div(cu.hr);
+      pages = p.paged ? pdiv.div(cu.L + p.page_size - 1) : 0;
     }
+    const TileBoxes tb = tile_boxes(p, cu, win, lane, h, pages, pdiv);
+    const bool draft = tb.draft;
     const int hf = lane & 1, i = lane >> 1;  // this lane's box: 64-dim half, row group
-    int y = 0;
-    if (draft) y = (cu.c * p.hkv + h) * p.n_max + key0 + i * br;
-    else if (p.paged) y = (pid * p.hkv + h) * p.page_size + ((key0 + i * br) % p.page_size);
-    else y = (cu.c * p.hkv + h) * p.l_cap + key0;
-    const uint32_t tx = nbox * br * 128 * 2;  // bytes of one K (or V) tile's boxes
+    const uint32_t tx = tb.nbox * tb.br * 128 * 2;  // bytes of one K (or V) tile's boxes
     int ok = 1;
     if (kv == 0 && (cu.t == cu.t_begin || cu.lt == 0)) {  // first tile of a piece: the unit's q block
       if (lane == 0) {
@@ -647,17 +673,22 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
       const int slot = kv ? t % kNV : t % kNK;
       const int round = kv ? t / kNV : t / kNK;
       uint64_t* fullb = kv ? &sm.vfull[slot] : &sm.kfull[slot];
-      uint64_t* emptyb = kv ? &sm.vempty[slot] : &sm.kempty[slot];
-      if (lane == 0 && ok) ok = mbar_wait(smem_addr(emptyb), (round & 1) ^ 1u, p.err) && !*pipe.abort;
+      // A V slot is free once P.V of its previous tile completed, a K slot once
+      // QK^T of its previous tile (t - kNK) completed.
+      if (lane == 0 && ok) {
+        if (kv) ok = mbar_wait(smem_addr(&sm.vempty[slot]), (round & 1) ^ 1u, p.err);
+        else if (t >= kNK) ok = mbar_wait(smem_addr(&sm.sfull[(t - kNK) % kNS]), ((t - kNK) / kNS) & 1, p.err);
+        ok = ok && !*pipe.abort;
+      }
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (ok) {
         const uint32_t full_bar = smem_addr(fullb);
         if (lane == 0) mbar_arrive_expect_tx(full_bar, tx);
-        if (i < nbox) {
+        if (i < tb.nbox) {
           const uint32_t dst = smem_addr((kv ? sm.vring : sm.kring) + static_cast<size_t>(slot) * kKVBytes) +
-                               hf * kHalfBytes + i * br * 128;
+                               hf * kHalfBytes + i * tb.br * 128;
           const CUtensorMap* map = draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
-          tma_load_2d(dst, map, hf * 64, y, full_bar, policy);
+          tma_load_2d(dst, map, hf * 64, tb.y, full_bar, policy);
         }
         if (lane == 0) sm.misc[kv ? 5 : 1] = t + 1;
       }
@@ -678,23 +709,24 @@ __global__ void __launch_bounds__(kThreads, 1)
   const Smem sm = carve(smem_raw, p.C);
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kNK; ++s) {
-      mbar_init(smem_addr(&sm.kfull[s]), 1);
-      mbar_init(smem_addr(&sm.kempty[s]), 1);
-    }
+    for (int s = 0; s < kNK; ++s) mbar_init(smem_addr(&sm.kfull[s]), 1);
     for (int s = 0; s < kNV; ++s) {
       mbar_init(smem_addr(&sm.vfull[s]), 1);
       mbar_init(smem_addr(&sm.vempty[s]), 1);
     }
     mbar_init(smem_addr(sm.qfull), 1);
     mbar_init(smem_addr(sm.qempty), 1);
-    for (int b = 0; b < kNS; ++b) mbar_init(smem_addr(&sm.sfull[b]), 1);
+    for (int b = 0; b < kNS; ++b) {
+      mbar_init(smem_addr(&sm.sfull[b]), 1);
+      mbar_init(smem_addr(&sm.sfree[b]), kSoftmaxThreads / 2);
+    }
     for (int b = 0; b < kNP; ++b) {
       mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads / 2);
       mbar_init(smem_addr(&sm.pvdone[b]), 1);
     }
     mbar_init(smem_addr(sm.ofree), kSoftmaxThreads);
-    mbar_init(smem_addr(sm.mmadone), 1);
+    mbar_init(smem_addr(&sm.mmadone[0]), 1);
+    mbar_init(smem_addr(&sm.mmadone[1]), 1);
     for (int i = 0; i < 8; ++i) sm.misc[i] = 0;
     fence_mbar_init();
     prefetch_tensormap(&maps.tk);
@@ -715,11 +747,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
   if (warp == kProducerWarp || warp == kProducerVWarp) {
     run_producer_tc<kSpread>(p, maps, sm, pipe, cu, nq_box, warp == kProducerVWarp ? 1 : 0);
-  } else if (warp == kMmaWarp) {
+  } else if (warp == kMmaWarp || warp == kMmaPvWarp) {
+    const int stream = warp == kMmaWarp ? 0 : 1;
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
-      run_mma(p, sm, pipe, tmem, cu);
+      if (stream == 0) run_mma_qk(p, sm, pipe, tmem, cu);
+      else run_mma_pv(p, sm, pipe, tmem, cu);
       // Every MMA must have completed before TMEM is released.
-      mbar_wait(smem_addr(sm.mmadone), 0, p.err);
+      mbar_wait(smem_addr(&sm.mmadone[stream]), 0, p.err);
     }
     __syncwarp();
   } else if (warp < 8) {
