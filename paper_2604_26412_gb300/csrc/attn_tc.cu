@@ -7,8 +7,8 @@
 //   S = Q K^T      tcgen05.mma M=128 N=64  K=128 (8 x K16), A = Q (smem), B = K tile (smem), D = S (TMEM)
 //   P = softmax(S) one thread per row: TMEM -> registers -> bf16 P (smem, 128B-swizzled)
 //   O += P V       tcgen05.mma M=128 N=128 K=64 (4 x K16), A = P (smem), B = V tile (smem, MN-major), D = O (TMEM)
-// Warp roles: warps 0..7 are two softmax warpgroups; warp 10 loads K tiles
-// and the q block of each piece by TMA, warp 9 loads V tiles (a single warp
+// Warp roles: warps 0..7 are two softmax warpgroups; warps 10 and 9 load the
+// K and V tiles (and q blocks) of even and odd tiles by TMA (a single warp
 // keeps too few bulk-tensor loads in flight to reach full HBM bandwidth);
 // warp 11 owns TMEM and one of its threads issues every QK^T, one thread of
 // warp 8 every P.V.
@@ -33,8 +33,8 @@ constexpr int kKVBytes = kKVTileBytes;     // one K or V tile
 constexpr int kNS = 4;                     // S buffers in TMEM: QK^T may run up to 4 tiles ahead of P.V
 constexpr int kNP = 3;                     // P buffers in shared memory
 constexpr int kThreads = 12 * 32;
-constexpr int kProducerWarp = 10;          // K ring and q blocks
-constexpr int kProducerVWarp = 9;          // V ring
+constexpr int kProducerWarp = 10;          // K, V and q loads of even tiles
+constexpr int kProducerVWarp = 9;          // K, V and q loads of odd tiles
 constexpr int kMmaWarp = 11;               // TMEM owner, QK^T issuer
 constexpr int kMmaPvWarp = 8;              // P.V issuer
 constexpr int kSoftmaxThreads = 256;       // two warpgroups
@@ -42,6 +42,7 @@ constexpr int kBarSoftmax = 1;             // named barrier among the softmax wa
 constexpr int kPBufBytes = kQRows * 128;   // 128 rows x 64 keys bf16
 constexpr uint32_t kTmemCols = 512;        // S0..S3 [0,256), O0 [256,384), O1 [384,512)
 constexpr uint32_t kTmemO = kNS * kTileKeys;
+constexpr int kMiscInts = 12;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max grows by > 256x
 
 // ------------------------------------------------------------ tcgen05 wrappers
@@ -185,7 +186,8 @@ struct Smem {
   int* par;            // [64]
   float* comb;         // [128][2] second warpgroup's (max, sum) per row at a piece end
   uint32_t* tmem_base;
-  int* misc;           // [0] abort, [1]/[2] K tiles issued/consumed, [3]/[4] q blocks, [5]/[6] V tiles
+  int* misc;           // [0] abort, [2] K tiles consumed, [3]/[4] q blocks issued/consumed, [6] V tiles consumed,
+                       // [8..9] / [10..11] K / V tiles issued per producer warp
   int* len;
   int* base;
 };
@@ -195,7 +197,7 @@ __host__ __device__ inline size_t smem_bytes(int C) {
   off += sizeof(uint64_t) * (kNK + 2 * kNV + 2 + 2 * kNS + 2 * kNP + 3);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(float) * 2 * kQRows;
-  off += sizeof(uint32_t) * 4 + sizeof(int) * 8;
+  off += sizeof(uint32_t) * 4 + sizeof(int) * kMiscInts;
   off += sizeof(int) * (2 * C + 1);
   return off + 1024;
 }
@@ -228,7 +230,7 @@ __device__ Smem carve(uint8_t* raw, int C) {
   s.comb = reinterpret_cast<float*>(s.par + kMaxTreeNodes);
   s.tmem_base = reinterpret_cast<uint32_t*>(s.comb + 2 * kQRows);
   s.misc = reinterpret_cast<int*>(s.tmem_base + 4);
-  s.len = s.misc + 8;
+  s.len = s.misc + kMiscInts;
   s.base = s.len + C;
   return s;
 }
@@ -484,8 +486,14 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       mbar_arrive(smem_addr(&sm.pfull[b]));
     }
     if (ti.last) {
-      const int b = t % kNP;
-      bool ok = live && mbar_wait(smem_addr(&sm.pvdone[b]), (t / kNP) & 1, p.err);
+      // Every P.V of the piece has completed once P.V of tile t has (P.V
+      // completes in tile order).  The warpgroup that does not own tile t last
+      // waited P.V of tile t - 4, too far back to tell tile t's phase of pvdone
+      // from tile t - 6's by parity, so it first waits P.V of its own tile t - 1.
+      bool ok = live;
+      if (ok && (t & 1) != wg && t >= 1)
+        ok = mbar_wait(smem_addr(&sm.pvdone[(t - 1) % kNP]), ((t - 1) / kNP) & 1, p.err);
+      ok = ok && mbar_wait(smem_addr(&sm.pvdone[t % kNP]), (t / kNP) & 1, p.err);
       ok = __all_sync(0xffffffffu, ok);
       tc_fence_after();
       float l_row = l_run;
@@ -496,6 +504,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         sm.comb[2 * tl + 1] = l_row;
       }
       named_barrier_sync(kBarSoftmax, kSoftmaxThreads);
+      tc_fence_after();
       if (wg == 0 && ok && warp_live) {
         const float m1 = sm.comb[2 * tl], l1 = sm.comb[2 * tl + 1];
         const float M = fmaxf(m_run, m1);
@@ -618,15 +627,23 @@ __device__ __forceinline__ TileBoxes tile_boxes(const AttnParams& p, const Curso
   return tb;
 }
 
-// Walks this CTA's tiles and loads one of the two rings, each box from its
-// own lane: role 0 loads the K ring and one q block per piece (single
-// buffer), role 1 the V ring.  Two producer warps keep twice the loads in
-// flight that one warp can (a warp's bulk-tensor issues stall while its
-// earlier ones are outstanding).  A spread unit's q block goes in boxes of 16
-// stacked rows, box k to TMEM lanes (= q buffer rows) 32 k .. 32 k + 15.
+// Walks this CTA's tiles and loads those with t % 2 == role: their K tile
+// into the K ring and their V tile into the V ring, each box from its own
+// lane.  Two producer warps keep twice the loads in flight that one warp can
+// (a warp's bulk-tensor issues stall while its earlier ones are outstanding),
+// and each tile's page lookups are done once for both rings.
+// The q block of every piece (single buffer) is loaded by role 0 alone: an
+// mbarrier wait by parity cannot tell a phase from the one two phases
+// earlier, so the q-buffer release must be waited by a thread that also
+// waited its previous phase.  (A ring slot is safe to wait from either warp:
+// its release is an in-order MMA completion that the warp's own previous
+// wait already covers two phases back.)  A spread unit's q block goes in
+// boxes of 16 stacked rows, box k to TMEM lanes (= q buffer rows)
+// 32 k .. 32 k + 15.  misc[8 + role] / misc[10 + role]: one past the last K /
+// V tile this warp issued (read by the drain after an abort).
 template <bool kSpread>
 __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const TensorMaps& maps, const Smem& sm,
-                                                const Pipe& pipe, Cursor cu, int nq_box, int kv) {
+                                                const Pipe& pipe, Cursor cu, int nq_box, int role) {
   const int lane = threadIdx.x & 31;
   const uint64_t policy = l2_policy_evict_first();
   PageWindow win;
@@ -635,19 +652,21 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
   const bool small = p.len_bound < (1 << 24) - 2 * kTileKeys;
   const FastDiv pdiv(p.paged ? p.page_size : 1, small), rbdiv(p.row_blocks, true);
   int unit_c = -1, unit_hr = -1, h = 0, pages = 0;  // the current unit's KV head and its cache's pages
-  while (cu.t < cu.t_end) {
+  int ok = 1;
+  for (; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
+    const bool first = cu.t == cu.t_begin || cu.lt == 0;  // first tile of a piece
+    const bool mine = (t & 1) == role;
+    if (!mine && !(first && role == 0)) {
+      piece += first;
+      continue;
+    }
     if (cu.c != unit_c || cu.hr != unit_hr) {
       unit_c = cu.c;
       unit_hr = cu.hr;
       h = rbdiv.div(cu.hr);
       pages = p.paged ? pdiv.div(cu.L + p.page_size - 1) : 0;
     }
-    const TileBoxes tb = tile_boxes(p, cu, win, lane, h, pages, pdiv);
-    const bool draft = tb.draft;
-    const int hf = lane & 1, i = lane >> 1;  // this lane's box: 64-dim half, row group
-    const uint32_t tx = tb.nbox * tb.br * 128 * 2;  // bytes of one K (or V) tile's boxes
-    int ok = 1;
-    if (kv == 0 && (cu.t == cu.t_begin || cu.lt == 0)) {  // first tile of a piece: the unit's q block
+    if (first && role == 0) {  // the unit's q block
       if (lane == 0) {
         const uint32_t qbar = smem_addr(sm.qfull);
         ok = mbar_wait(smem_addr(sm.qempty), (piece & 1) ^ 1u, p.err) && !*pipe.abort;
@@ -667,38 +686,43 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
           sm.misc[3] = piece + 1;
         }
       }
-      ++piece;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) *pipe.abort = 1;
+        break;
+      }
     }
-    {
+    piece += first;
+    if (!mine) continue;
+    const TileBoxes tb = tile_boxes(p, cu, win, lane, h, pages, pdiv);
+    const int hf = lane & 1, i = lane >> 1;  // this lane's box: 64-dim half, row group
+    const uint32_t tx = tb.nbox * tb.br * 128 * 2;  // bytes of one K (or V) tile's boxes
+#pragma unroll
+    for (int kv = 0; kv < 2; ++kv) {
       const int slot = kv ? t % kNV : t % kNK;
-      const int round = kv ? t / kNV : t / kNK;
-      uint64_t* fullb = kv ? &sm.vfull[slot] : &sm.kfull[slot];
       // A V slot is free once P.V of its previous tile completed, a K slot once
       // QK^T of its previous tile (t - kNK) completed.
       if (lane == 0 && ok) {
-        if (kv) ok = mbar_wait(smem_addr(&sm.vempty[slot]), (round & 1) ^ 1u, p.err);
+        if (kv) ok = mbar_wait(smem_addr(&sm.vempty[slot]), ((t / kNV) & 1) ^ 1u, p.err);
         else if (t >= kNK) ok = mbar_wait(smem_addr(&sm.sfull[(t - kNK) % kNS]), ((t - kNK) / kNS) & 1, p.err);
         ok = ok && !*pipe.abort;
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (ok) {
-        const uint32_t full_bar = smem_addr(fullb);
-        if (lane == 0) mbar_arrive_expect_tx(full_bar, tx);
-        if (i < tb.nbox) {
-          const uint32_t dst = smem_addr((kv ? sm.vring : sm.kring) + static_cast<size_t>(slot) * kKVBytes) +
-                               hf * kHalfBytes + i * tb.br * 128;
-          const CUtensorMap* map = draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
-          tma_load_2d(dst, map, hf * 64, tb.y, full_bar, policy);
-        }
-        if (lane == 0) sm.misc[kv ? 5 : 1] = t + 1;
+      if (!ok) break;
+      const uint32_t full_bar = smem_addr(kv ? &sm.vfull[slot] : &sm.kfull[slot]);
+      if (lane == 0) mbar_arrive_expect_tx(full_bar, tx);
+      if (i < tb.nbox) {
+        const uint32_t dst = smem_addr((kv ? sm.vring : sm.kring) + static_cast<size_t>(slot) * kKVBytes) +
+                             hf * kHalfBytes + i * tb.br * 128;
+        const CUtensorMap* map = tb.draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
+        tma_load_2d(dst, map, hf * 64, tb.y, full_bar, policy);
       }
+      if (lane == 0) sm.misc[(kv ? 10 : 8) + role] = t + 1;
     }
     if (!ok) {
       if (lane == 0) *pipe.abort = 1;
       break;
     }
-    ++t;
-    cursor_next(cu, p, sm.len);
   }
 }
 
@@ -727,7 +751,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(smem_addr(sm.ofree), kSoftmaxThreads);
     mbar_init(smem_addr(&sm.mmadone[0]), 1);
     mbar_init(smem_addr(&sm.mmadone[1]), 1);
-    for (int i = 0; i < 8; ++i) sm.misc[i] = 0;
+    for (int i = 0; i < kMiscInts; ++i) sm.misc[i] = 0;
     fence_mbar_init();
     prefetch_tensormap(&maps.tk);
     prefetch_tensormap(&maps.tv);
@@ -744,9 +768,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *sm.tmem_base;
   const Cursor cu = cursor_begin(p, sm.len, sm.base);
-  Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
+  Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), nullptr};
   if (warp == kProducerWarp || warp == kProducerVWarp) {
-    run_producer_tc<kSpread>(p, maps, sm, pipe, cu, nq_box, warp == kProducerVWarp ? 1 : 0);
+    run_producer_tc<kSpread>(p, maps, sm, pipe, cu, nq_box, warp == kProducerWarp ? 0 : 1);
   } else if (warp == kMmaWarp || warp == kMmaPvWarp) {
     const int stream = warp == kMmaWarp ? 0 : 1;
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
@@ -764,10 +788,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   if (threadIdx.x == 0 && *pipe.abort) {
     // A wait timed out: let every TMA load still in flight land before the CTA exits.
-    for (int k = sm.misc[2]; k < sm.misc[1]; ++k)
-      if (!mbar_wait(smem_addr(&sm.kfull[k % kNK]), (k / kNK) & 1, p.err)) break;
-    for (int k = sm.misc[6]; k < sm.misc[5]; ++k)
-      if (!mbar_wait(smem_addr(&sm.vfull[k % kNV]), (k / kNV) & 1, p.err)) break;
+    // Tile k was loaded by producer warp k % 2, which issues its tiles in order.
+    for (int k = sm.misc[2]; k < max(sm.misc[8], sm.misc[9]); ++k)
+      if (k < sm.misc[8 + (k & 1)] && !mbar_wait(smem_addr(&sm.kfull[k % kNK]), (k / kNK) & 1, p.err)) break;
+    for (int k = sm.misc[6]; k < max(sm.misc[10], sm.misc[11]); ++k)
+      if (k < sm.misc[10 + (k & 1)] && !mbar_wait(smem_addr(&sm.vfull[k % kNV]), (k / kNV) & 1, p.err)) break;
     for (int k = sm.misc[4]; k < sm.misc[3]; ++k)
       if (!mbar_wait(smem_addr(sm.qfull), k & 1, p.err)) break;
   }
