@@ -31,7 +31,7 @@ def _case(lens, levels, tree, paged, page_size=16, hq=32, hkv=8, n_query=None, s
     return spec, inp, dk, dv, q, N, Nq
 
 
-def _run(spec, inp, dk, dv, q, N, Nq, flags=0, num_ctas=0, scale=0.0, parents=None):
+def _run(spec, inp, dk, dv, q, N, Nq, flags=0, num_ctas=0, scale=0.0, parents=None, ws=None):
     paged = inp.page_table is not None
     out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device="cuda")
     lse = torch.full(q.shape[:3], float("nan"), dtype=torch.float32, device="cuda")
@@ -44,8 +44,10 @@ def _run(spec, inp, dk, dv, q, N, Nq, flags=0, num_ctas=0, scale=0.0, parents=No
                          flags=flags, num_ctas=num_ctas, err_flag=err)
     ws_bytes = kvshot.workspace_size(d)
     assert ws_bytes > 0
-    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
-    d.workspace, d.workspace_bytes = ws.data_ptr(), ws_bytes
+    if ws is None:
+        ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    assert ws.numel() >= ws_bytes
+    d.workspace, d.workspace_bytes = ws.data_ptr(), ws.numel()
     par = (inp.tree_parent[:, :N].contiguous() if parents is None else parents)
     kvshot.draft_attn(d, q, inp.target_k, inp.target_v, inp.page_table, inp.seq_lens, dk, dv, par, out, lse)
     torch.cuda.synchronize()
@@ -196,3 +198,23 @@ def test_workspace_too_small_is_rejected():
     st = kvshot.draft_attn_status(d, q, inp.target_k, inp.target_v, inp.page_table, inp.seq_lens, dk, dv,
                                   inp.tree_parent[:, :N].contiguous(), out, lse)
     assert st == kvshot.KVSHOT_ERR_WORKSPACE
+
+
+def test_one_workspace_serves_successive_calls_and_shapes():
+    """One workspace is reused by successive calls of different shapes and grids (units split into
+    pieces that straddle CTAs and are merged): no call depends on what an earlier one left in it."""
+    cases = [((3000, 517, 64), (4, 4, 4), True, True, 16, 32, 8, 12),   # 48 rows (spread), 3 caches
+             ((700, 1300), (8, 12, 12), True, True, 64, 32, 8, 32),     # 128 rows (dense)
+             ((250, 70), (1, 1, 1), False, True, 16, 32, 1, 2)]          # G = 32, contiguous
+    prepared = []
+    for k, (lens, levels, tree, paged, P, hq, hkv, nq) in enumerate(cases):
+        spec, inp, dk, dv, q, N, Nq = _case(lens, levels, tree, paged, P, hq, hkv, nq, seed=100 + k)
+        ref = gh.oracle_attn(gh.HostCache(inp), q, dk, dv, N, Nq)
+        prepared.append((spec, inp, dk, dv, q, N, Nq, ref))
+    ws = torch.full((64 << 20,), 0x7F, dtype=torch.uint8, device="cuda")  # not zero: nothing may be assumed
+    for rep in range(2):
+        for k, (spec, inp, dk, dv, q, N, Nq, (ref_out, ref_lse)) in enumerate(prepared):
+            for flags in (kvshot.KVSHOT_FORCE_TC, kvshot.KVSHOT_FORCE_MMA):
+                for num_ctas in (7, 3, 0):
+                    out, lse = _run(spec, inp, dk, dv, q, N, Nq, flags=flags, num_ctas=num_ctas, ws=ws)
+                    gh.compare(out, lse, ref_out, ref_lse, f"shared workspace rep {rep} case {k} flags {flags} ctas {num_ctas}")
