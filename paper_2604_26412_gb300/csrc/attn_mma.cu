@@ -347,6 +347,7 @@ template <class CF>
 __global__ void __launch_bounds__(CF::kThreads, CF::kMinBlocks)
     attn_mma_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ TensorMaps maps) {
   extern __shared__ uint8_t smem_raw[];
+  if (threadIdx.x == 0) allow_dependent_launch();  // the merge may be scheduled as CTAs finish
   const Smem sm = carve<CF>(smem_raw, p.C);
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {

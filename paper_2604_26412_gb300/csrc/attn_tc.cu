@@ -730,6 +730,7 @@ template <bool kSpread>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ TensorMaps maps, int nq_box) {
   extern __shared__ uint8_t smem_raw[];
+  if (threadIdx.x == 0) allow_dependent_launch();  // the merge may be scheduled as CTAs finish
   const Smem sm = carve(smem_raw, p.C);
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {

@@ -93,6 +93,16 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
   return done != 0;
 }
 
+// Programmatic dependent launch.  The attention kernels let the kernel that
+// follows them in the stream (the split merge, launched with programmatic
+// stream serialization) be scheduled onto SMs as attention CTAs finish; that
+// kernel waits for the whole attention grid to complete, memory included,
+// before it reads anything, so only the launch latency is hidden.
+__device__ __forceinline__ void allow_dependent_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void wait_for_prerequisite_grid() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ uint64_t l2_policy_evict_first() {
   uint64_t pol;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));

@@ -14,11 +14,15 @@ using namespace dev;
 
 constexpr int kMergeThreads = 256;
 constexpr int kMergeRows = kMergeThreads / 32;  // rows per CTA, one warp per row
+constexpr int kMergeBatch = 4;                  // pieces whose outputs are loaded in one batch
 
 // Workspace slot of the piece computed by CTA b is u + b.  One warp per row
-// of a unit; lane k reads the lse of piece b0 + k, and every piece's partial
-// output (lane = 4 dims) is read in one batch of independent loads.
+// of a unit.  Launched behind the attention kernel with programmatic stream
+// serialization: it waits for that grid first.  Then two rounds of loads: the
+// plan (length, tile prefix), then every piece's lse (lane k: piece b0 + k)
+// together with the first kMergeBatch pieces' outputs (lane: 4 dims).
 __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_constant__ AttnParams p) {
+  wait_for_prerequisite_grid();
   const int blocks_per_unit = (p.rows_per_unit + kMergeRows - 1) / kMergeRows;
   const int u = blockIdx.x / blocks_per_unit;
   const int r = (blockIdx.x - u * blocks_per_unit) * kMergeRows + (threadIdx.x >> 5);
@@ -35,35 +39,47 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
   const int b0 = gs / tpc, b1 = (gs + ut - 1) / tpc;
   if (b0 == b1) return;  // the unit lived in one CTA, which wrote the output itself
   const int np = b1 - b0 + 1;
-  // Pass 1: the largest piece lse.
-  float M = -INFINITY;
-  for (int k = lane; k < np; k += 32)
-    M = fmaxf(M, p.ws_lse[static_cast<size_t>(u + b0 + k) * p.rows_per_unit + r]);
+  const size_t row0 = static_cast<size_t>(u + b0) * p.rows_per_unit + r;  // piece k's row: row0 + k * rows
+  float ls = lane < np ? p.ws_lse[row0 + static_cast<size_t>(lane) * p.rows_per_unit] : -INFINITY;
+  float4 v[kMergeBatch];
+#pragma unroll
+  for (int k = 0; k < kMergeBatch; ++k)
+    v[k] = k < np ? *reinterpret_cast<const float4*>(p.ws_o + (row0 + static_cast<size_t>(k) * p.rows_per_unit) *
+                                                                   kHeadDim + 4 * lane)
+                  : make_float4(0.f, 0.f, 0.f, 0.f);
+  float M = ls;
+  for (int k = lane + 32; k < np; k += 32)  // more than 32 pieces: fold the rest into this lane's max
+    M = fmaxf(M, p.ws_lse[row0 + static_cast<size_t>(k) * p.rows_per_unit]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  // Pass 2: weights e^(lse_s - M) and the weighted partial outputs.
   float Lsum = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   if (M != -INFINITY) {
     for (int k0 = 0; k0 < np; k0 += 32) {
-      const int k = k0 + lane;
       float wl = 0.f;
-      if (k < np) {
-        const float ls = p.ws_lse[static_cast<size_t>(u + b0 + k) * p.rows_per_unit + r];
-        wl = ls == -INFINITY ? 0.f : exp2f(ls - M);
+      if (k0 + lane < np) {
+        const float lk = k0 == 0 ? ls : p.ws_lse[row0 + static_cast<size_t>(k0 + lane) * p.rows_per_unit];
+        wl = lk == -INFINITY ? 0.f : exp2f(lk - M);
       }
       const int n = min(32, np - k0);
       for (int j = 0; j < n; ++j) {
         const float w = __shfl_sync(0xffffffffu, wl, j);
         Lsum += w;
-        if (w != 0.f) {
-          const size_t row = static_cast<size_t>(u + b0 + k0 + j) * p.rows_per_unit + r;
-          const float4 v = *reinterpret_cast<const float4*>(p.ws_o + row * kHeadDim + 4 * lane);
-          acc.x += w * v.x;
-          acc.y += w * v.y;
-          acc.z += w * v.z;
-          acc.w += w * v.w;
+        const int k = k0 + j;
+        float4 x;
+        if (k < kMergeBatch) {
+          x = v[0];
+#pragma unroll
+          for (int q = 1; q < kMergeBatch; ++q)
+            if (k == q) x = v[q];
+        } else {
+          x = *reinterpret_cast<const float4*>(p.ws_o + (row0 + static_cast<size_t>(k) * p.rows_per_unit) * kHeadDim +
+                                                4 * lane);
         }
+        acc.x += w * x.x;
+        acc.y += w * x.y;
+        acc.z += w * x.z;
+        acc.w += w * x.w;
       }
     }
   }
@@ -167,8 +183,17 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(const __grid_con
 cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream) {
   const int units = p.C * p.hkv * p.row_blocks;
   const int blocks = units * ((p.rows_per_unit + kMergeRows - 1) / kMergeRows);
-  merge_kernel<<<blocks, kMergeThreads, 0, stream>>>(p);
-  return cudaGetLastError();
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(blocks);
+  cfg.blockDim = dim3(kMergeThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, merge_kernel, p);
 }
 
 cudaError_t launch_append(const AppendParams& a, cudaStream_t stream) {
