@@ -588,9 +588,9 @@ struct FastDiv {
   }
 };
 
-// TMA boxes of one K (or V) tile: `nbox` boxes of `br` rows in each 64-dim
-// half; lane (hf = lane & 1, i = lane >> 1) owns box i of half hf, whose first
-// row in the tile's tensor map (target or draft) is y.  h is the unit's KV
+// TMA boxes of one K (or V) tile: `nbox` (<= 8) boxes of `br` rows in each
+// 64-dim half; lanes l and l + 16 (hf = l & 1, i = (l & 15) >> 1) own box i of
+// half hf, whose first row in the tile's tensor map (target or draft) is y.  h is the unit's KV
 // head, `pages` the cache's pages in use.  Warp-wide.
 struct TileBoxes {
   bool draft;
@@ -603,7 +603,7 @@ __device__ __forceinline__ TileBoxes tile_boxes(const AttnParams& p, const Curso
   tb.draft = cu.lt >= cu.pt;
   const int key0 = (tb.draft ? cu.lt - cu.pt : cu.lt) * kTileKeys;
   const int nkeys = min(kTileKeys, (tb.draft ? p.N : cu.L) - key0);
-  const int i = lane >> 1;
+  const int i = (lane & 15) >> 1;
   if (tb.draft) {
     tb.br = kDraftBoxRows;
     tb.nbox = (nkeys + kDraftBoxRows - 1) / kDraftBoxRows;
@@ -695,29 +695,35 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
     piece += first;
     if (!mine) continue;
     const TileBoxes tb = tile_boxes(p, cu, win, lane, h, pages, pdiv);
-    const int hf = lane & 1, i = lane >> 1;  // this lane's box: 64-dim half, row group
+    // Lanes 0..15 load the K boxes, lanes 16..31 the V boxes (half = lane & 1, row group = (lane & 15) >> 1).
+    const int kv = lane >> 4, hf = lane & 1, i = (lane & 15) >> 1;
     const uint32_t tx = tb.nbox * tb.br * 128 * 2;  // bytes of one K (or V) tile's boxes
-#pragma unroll
-    for (int kv = 0; kv < 2; ++kv) {
-      const int slot = kv ? t % kNV : t % kNK;
-      // A V slot is free once P.V of its previous tile completed, a K slot once
-      // QK^T of its previous tile (t - kNK) completed.
-      if (lane == 0 && ok) {
-        if (kv) ok = mbar_wait(smem_addr(&sm.vempty[slot]), ((t / kNV) & 1) ^ 1u, p.err);
-        else if (t >= kNK) ok = mbar_wait(smem_addr(&sm.sfull[(t - kNK) % kNS]), ((t - kNK) / kNS) & 1, p.err);
-        ok = ok && !*pipe.abort;
-      }
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) break;
-      const uint32_t full_bar = smem_addr(kv ? &sm.vfull[slot] : &sm.kfull[slot]);
-      if (lane == 0) mbar_arrive_expect_tx(full_bar, tx);
-      if (i < tb.nbox) {
-        const uint32_t dst = smem_addr((kv ? sm.vring : sm.kring) + static_cast<size_t>(slot) * kKVBytes) +
-                             hf * kHalfBytes + i * tb.br * 128;
-        const CUtensorMap* map = tb.draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
-        tma_load_2d(dst, map, hf * 64, tb.y, full_bar, policy);
-      }
-      if (lane == 0) sm.misc[(kv ? 10 : 8) + role] = t + 1;
+    const int kslot = t % kNK, vslot = t % kNV;
+    // A V slot is free once P.V of its previous tile completed, a K slot once QK^T of its previous tile
+    // (t - kNK) completed.  Lane 0 waits for the K slot and lane 1 for the V slot together.
+    if (lane < 2 && ok) {
+      const bool need = lane == 1 || t >= kNK;
+      const uint32_t bar = lane == 0 ? smem_addr(&sm.sfull[(t - kNK) % kNS]) : smem_addr(&sm.vempty[vslot]);
+      const uint32_t par = lane == 0 ? (((t - kNK) / kNS) & 1) : (((t / kNV) & 1) ^ 1u);
+      ok = (!need || mbar_wait(bar, par, p.err)) && !*pipe.abort;
+    }
+    ok = __all_sync(0xffffffffu, ok);
+    if (!ok) {
+      if (lane == 0) *pipe.abort = 1;
+      break;
+    }
+    const uint32_t full_bar = smem_addr(kv ? &sm.vfull[vslot] : &sm.kfull[kslot]);
+    if ((lane & 15) == 0) mbar_arrive_expect_tx(full_bar, tx);
+    if (i < tb.nbox) {
+      const uint32_t dst = smem_addr((kv ? sm.vring + static_cast<size_t>(vslot) * kKVBytes
+                                         : sm.kring + static_cast<size_t>(kslot) * kKVBytes)) +
+                           hf * kHalfBytes + i * tb.br * 128;
+      const CUtensorMap* map = tb.draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
+      tma_load_2d(dst, map, hf * 64, tb.y, full_bar, policy);
+    }
+    if (lane == 0) {
+      sm.misc[8 + role] = t + 1;
+      sm.misc[10 + role] = t + 1;
     }
     if (!ok) {
       if (lane == 0) *pipe.abort = 1;
