@@ -8,8 +8,9 @@
 //   P = softmax(S) one thread per row: TMEM -> registers -> bf16 P (smem, 128B-swizzled)
 //   O += P V       tcgen05.mma M=128 N=128 K=64 (4 x K16), A = P (smem), B = V tile (smem, MN-major), D = O (TMEM)
 // Warp roles: warps 0..7 are two softmax warpgroups; warps 10 and 9 load the
-// K and V tiles (and q blocks) of even and odd tiles by TMA (a single warp
-// keeps too few bulk-tensor loads in flight to reach full HBM bandwidth);
+// K and V tiles of even and odd tiles by TMA, warp 9 also the q blocks (a
+// single warp keeps too few bulk-tensor loads in flight to reach full HBM
+// bandwidth);
 // warp 11 owns TMEM and one of its threads issues every QK^T, one thread of
 // warp 8 every P.V.
 // Warpgroup w owns the tiles t with t % 2 == w: it turns S into P for all 64
@@ -33,8 +34,8 @@ constexpr int kKVBytes = kKVTileBytes;     // one K or V tile
 constexpr int kNS = 4;                     // S buffers in TMEM: QK^T may run up to 4 tiles ahead of P.V
 constexpr int kNP = 3;                     // P buffers in shared memory
 constexpr int kThreads = 12 * 32;
-constexpr int kProducerWarp = 10;          // K, V and q loads of even tiles
-constexpr int kProducerVWarp = 9;          // K, V and q loads of odd tiles
+constexpr int kProducerWarp = 10;          // K and V loads of even tiles
+constexpr int kProducerVWarp = 9;          // K and V loads of odd tiles, q blocks
 constexpr int kMmaWarp = 11;               // TMEM owner, QK^T issuer
 constexpr int kMmaPvWarp = 8;              // P.V issuer
 constexpr int kSoftmaxThreads = 256;       // two warpgroups
@@ -632,7 +633,8 @@ __device__ __forceinline__ TileBoxes tile_boxes(const AttnParams& p, const Curso
 // lane.  Two producer warps keep twice the loads in flight that one warp can
 // (a warp's bulk-tensor issues stall while its earlier ones are outstanding),
 // and each tile's page lookups are done once for both rings.
-// The q block of every piece (single buffer) is loaded by role 0 alone: an
+// The q block of every piece (single buffer) is loaded by role 1 alone (so the
+// first tile's K and V, from role 0, do not queue behind it): an
 // mbarrier wait by parity cannot tell a phase from the one two phases
 // earlier, so the q-buffer release must be waited by a thread that also
 // waited its previous phase.  (A ring slot is safe to wait from either warp:
@@ -656,7 +658,7 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
   for (; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
     const bool first = cu.t == cu.t_begin || cu.lt == 0;  // first tile of a piece
     const bool mine = (t & 1) == role;
-    if (!mine && !(first && role == 0)) {
+    if (!mine && !(first && role == 1)) {
       piece += first;
       continue;
     }
@@ -666,7 +668,7 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
       h = rbdiv.div(cu.hr);
       pages = p.paged ? pdiv.div(cu.L + p.page_size - 1) : 0;
     }
-    if (first && role == 0) {  // the unit's q block
+    if (first && role == 1) {  // the unit's q block
       if (lane == 0) {
         const uint32_t qbar = smem_addr(sm.qfull);
         ok = mbar_wait(smem_addr(sm.qempty), (piece & 1) ^ 1u, p.err) && !*pipe.abort;
