@@ -14,14 +14,15 @@ using namespace dev;
 
 constexpr int kMergeThreads = 256;
 constexpr int kMergeRows = kMergeThreads / 32;  // rows per CTA, one warp per row
-constexpr int kMergeBatch = 4;                  // pieces whose outputs are loaded in one batch
 
 // Workspace slot of the piece computed by CTA b is u + b.  One warp per row
 // of a unit.  Launched behind the attention kernel with programmatic stream
 // serialization: it waits for that grid first.  Then two rounds of loads: the
 // plan (length, tile prefix), then every piece's lse (lane k: piece b0 + k)
-// together with the first kMergeBatch pieces' outputs (lane: 4 dims).
-__global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_constant__ AttnParams p) {
+// together with the first two pieces' outputs (lane: 4 dims).
+// 6 resident CTAs per SM (<= 40 registers): a unit's rows for every split unit of the largest
+// per-level plans fit in one wave, so no merge CTA waits for another to finish.
+__global__ void __launch_bounds__(kMergeThreads, 6) merge_kernel(const __grid_constant__ AttnParams p) {
   wait_for_prerequisite_grid();
   const int blocks_per_unit = (p.rows_per_unit + kMergeRows - 1) / kMergeRows;
   const int u = blockIdx.x / blocks_per_unit;
@@ -39,14 +40,15 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
   const int b0 = gs / tpc, b1 = (gs + ut - 1) / tpc;
   if (b0 == b1) return;  // the unit lived in one CTA, which wrote the output itself
   const int np = b1 - b0 + 1;
+  const int nl = rr / p.G, g = rr - nl * p.G;
+  const size_t orow = (static_cast<size_t>(c) * p.Nq + nl) * p.hq + h * p.G + g;
   const size_t row0 = static_cast<size_t>(u + b0) * p.rows_per_unit + r;  // piece k's row: row0 + k * rows
   float ls = lane < np ? p.ws_lse[row0 + static_cast<size_t>(lane) * p.rows_per_unit] : -INFINITY;
-  float4 v[kMergeBatch];
-#pragma unroll
-  for (int k = 0; k < kMergeBatch; ++k)
-    v[k] = k < np ? *reinterpret_cast<const float4*>(p.ws_o + (row0 + static_cast<size_t>(k) * p.rows_per_unit) *
-                                                                   kHeadDim + 4 * lane)
-                  : make_float4(0.f, 0.f, 0.f, 0.f);
+  const int ostride = p.rows_per_unit * (kHeadDim / 4);  // float4s from one piece's row to the next's
+  const float4* op = reinterpret_cast<const float4*>(p.ws_o + row0 * kHeadDim) + lane;
+  const float4 v0 = op[0];  // np >= 2 here
+  const float4 v1 = op[ostride];
+  op += 2 * ostride;  // piece 2
   float M = ls;
   for (int k = lane + 32; k < np; k += 32)  // more than 32 pieces: fold the rest into this lane's max
     M = fmaxf(M, p.ws_lse[row0 + static_cast<size_t>(k) * p.rows_per_unit]);
@@ -66,15 +68,12 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
         const float w = __shfl_sync(0xffffffffu, wl, j);
         Lsum += w;
         const int k = k0 + j;
-        float4 x;
-        if (k < kMergeBatch) {
-          x = v[0];
-#pragma unroll
-          for (int q = 1; q < kMergeBatch; ++q)
-            if (k == q) x = v[q];
-        } else {
-          x = *reinterpret_cast<const float4*>(p.ws_o + (row0 + static_cast<size_t>(k) * p.rows_per_unit) * kHeadDim +
-                                                4 * lane);
+        float4 x = v0;
+        if (k == 1) {
+          x = v1;
+        } else if (k > 1) {
+          x = *op;
+          op += ostride;
         }
         acc.x += w * x.x;
         acc.y += w * x.y;
@@ -84,8 +83,6 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
     }
   }
   const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-  const int nl = rr / p.G, g = rr - nl * p.G;
-  const size_t orow = (static_cast<size_t>(c) * p.Nq + nl) * p.hq + h * p.G + g;
   uint2 packed;
   packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
   packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
