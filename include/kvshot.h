@@ -94,8 +94,7 @@ typedef struct kvshot_attn_desc {
 
 /*
  * Bytes of workspace kvshot_draft_attn needs for `desc` on the current device
- * (partial softmax states of work pieces that straddle CTAs, plus the work
- * plan).  Returns 0 if the descriptor is invalid.  The size depends on the
+ * (partial softmax states of work pieces that straddle CTAs).  Returns 0 if the descriptor is invalid.  The size depends on the
  * shape fields, flags, num_ctas and the device's SM count, not on pointers.
  */
 size_t kvshot_draft_attn_workspace_size(const kvshot_attn_desc* desc);

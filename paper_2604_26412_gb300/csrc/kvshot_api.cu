@@ -192,7 +192,7 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(grid, std::max<int64_t>(1, max_tiles))));
   pl->num_ctas = grid;
   const size_t slots = static_cast<size_t>(pl->units) + grid;
-  pl->off_lse = round_up(sizeof(int32_t) * (d->num_caches + 1), 256);
+  pl->off_lse = 0;
   pl->off_o = pl->off_lse + round_up(sizeof(float) * slots * pl->rows_per_unit, 256);
   pl->bytes = pl->off_o + sizeof(float) * slots * pl->rows_per_unit * kHeadDim;
   return KVSHOT_OK;
@@ -273,7 +273,6 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   p.tree_parent = tree_parent;
   p.err = d->err_flag;
   uint8_t* ws = static_cast<uint8_t*>(d->workspace);
-  p.ws_meta = reinterpret_cast<int32_t*>(ws);
   p.ws_lse = reinterpret_cast<float*>(ws + pl.off_lse);
   p.ws_o = reinterpret_cast<float*>(ws + pl.off_o);
   p.C = d->num_caches;

@@ -203,8 +203,7 @@ __device__ __forceinline__ int clamp_len(const AttnParams& p, int c) {
 }
 
 // s_len[c] = clamped L_c; s_base[c] = first global tile of cache c (prefix sum of
-// units x tiles per unit).  Whole block participates.  CTA 0 also publishes
-// s_base to the workspace for the merge kernel.
+// units x tiles per unit).  Whole block participates.
 __device__ __forceinline__ void build_plan(const AttnParams& p, int* s_len, int* s_base) {
   const int HR = p.hkv * p.row_blocks;
   for (int c = threadIdx.x; c < p.C; c += blockDim.x) {
@@ -230,8 +229,6 @@ __device__ __forceinline__ void build_plan(const AttnParams& p, int* s_len, int*
     if (lane == 0) s_base[0] = 0;
   }
   __syncthreads();
-  if (blockIdx.x == 0)
-    for (int c = threadIdx.x; c <= p.C; c += blockDim.x) p.ws_meta[c] = s_base[c];
 }
 
 // Tiles of CTA b: [b * tpc, min(T, (b + 1) * tpc)).

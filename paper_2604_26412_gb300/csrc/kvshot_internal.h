@@ -56,7 +56,6 @@ struct AttnParams {
   const int32_t* seq_lens;
   const int32_t* tree_parent;
   int32_t* err;             // may be null
-  int32_t* ws_meta;         // [C + 1] tile prefix per cache, written by CTA 0
   float* ws_lse;            // [slots, rows_per_unit] log2-domain lse of pieces
   float* ws_o;              // [slots, rows_per_unit, 128] normalised piece outputs
   int C, B, hq, hkv, G;

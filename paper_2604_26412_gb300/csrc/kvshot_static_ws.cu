@@ -58,8 +58,8 @@ extern "C" kvshot_status kvshot_draft_attn_static(const kvshot_attn_desc* desc, 
   if (need > kStaticBytes) return KVSHOT_ERR_WORKSPACE;
   void* scratch = nullptr;
   if (kvshot_status st = scratch_address(&scratch)) return st;
-  // The attention kernels write every scratch word they later read (the work
-  // plan first, then each piece's partial result before the merge reads it),
+  // The attention kernels write every scratch word they later read (each
+  // piece's partial result before the merge reads it),
   // so nothing in the array has to be cleared between calls.
   d.workspace = scratch;
   d.workspace_bytes = kStaticBytes;

@@ -17,13 +17,16 @@ constexpr int kMergeRows = kMergeThreads / 32;  // rows per CTA, one warp per ro
 
 // Workspace slot of the piece computed by CTA b is u + b.  One warp per row
 // of a unit.  Launched behind the attention kernel with programmatic stream
-// serialization: it waits for that grid first.  Then two rounds of loads: the
-// plan (length, tile prefix), then every piece's lse (lane k: piece b0 + k)
-// together with the first two pieces' outputs (lane: 4 dims).
+// serialization, so its CTAs start as the attention CTAs leave.  Each warp
+// first rebuilds the attention kernel's plan from the inputs alone (lengths ->
+// tiles per unit -> the unit's tile range -> the CTAs that held it): rows of
+// units that lived in one CTA leave at once, and the others only then wait
+// for the attention grid, with one round of loads left: every piece's lse
+// (lane k: piece b0 + k) together with the first two pieces' outputs (lane: 4
+// dims).
 // 6 resident CTAs per SM (<= 40 registers): a unit's rows for every split unit of the largest
 // per-level plans fit in one wave, so no merge CTA waits for another to finish.
 __global__ void __launch_bounds__(kMergeThreads, 6) merge_kernel(const __grid_constant__ AttnParams p) {
-  wait_for_prerequisite_grid();
   const int blocks_per_unit = (p.rows_per_unit + kMergeRows - 1) / kMergeRows;
   const int u = blockIdx.x / blocks_per_unit;
   const int r = (blockIdx.x - u * blocks_per_unit) * kMergeRows + (threadIdx.x >> 5);
@@ -33,12 +36,26 @@ __global__ void __launch_bounds__(kMergeThreads, 6) merge_kernel(const __grid_co
   const int h = hr / p.row_blocks, rb = hr - h * p.row_blocks;
   const int rr = rb * p.rows_per_unit + r;
   if (r >= p.rows_per_unit || rr >= p.rows_total) return;
-  const int L = clamp_len(p, c);
-  const int ut = (L + kTileKeys - 1) / kTileKeys + p.draft_tiles;
-  const int gs = p.ws_meta[c] + hr * ut;
-  const int tpc = tiles_per_cta(p.ws_meta[p.C], p.num_ctas);
+  // First tile of cache c and the total (the prefix sums of build_plan), 32 caches per round.
+  int cbase = 0, total = 0, ut = 0;
+  for (int c0 = 0; c0 < p.C; c0 += 32) {
+    const int cc = c0 + lane;
+    const int utc = cc < p.C ? (clamp_len(p, cc) + kTileKeys - 1) / kTileKeys + p.draft_tiles : 0;
+    int below = cc < c ? utc * HR : 0, all = utc * HR;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      below += __shfl_xor_sync(0xffffffffu, below, o);
+      all += __shfl_xor_sync(0xffffffffu, all, o);
+    }
+    cbase += below;
+    total += all;
+    if (c - c0 >= 0 && c - c0 < 32) ut = __shfl_sync(0xffffffffu, utc, c - c0);
+  }
+  const int gs = cbase + hr * ut;
+  const int tpc = tiles_per_cta(total, p.num_ctas);
   const int b0 = gs / tpc, b1 = (gs + ut - 1) / tpc;
   if (b0 == b1) return;  // the unit lived in one CTA, which wrote the output itself
+  wait_for_prerequisite_grid();
   const int np = b1 - b0 + 1;
   const int nl = rr / p.G, g = rr - nl * p.G;
   const size_t orow = (static_cast<size_t>(c) * p.Nq + nl) * p.hq + h * p.G + g;
