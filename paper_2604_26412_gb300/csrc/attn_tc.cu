@@ -739,8 +739,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ TensorMaps maps, int nq_box) {
   extern __shared__ uint8_t smem_raw[];
   if (threadIdx.x == 0) allow_dependent_launch();  // the merge may be scheduled as CTAs finish
+  // The plan's lengths are loaded first, so that their latency overlaps the set-up below
+  // (a negative length, invalid anyway, is clamped by the ordinary path).
+  const int len0 = static_cast<int>(threadIdx.x) < p.C ? p.seq_lens[threadIdx.x] : -1;
   const Smem sm = carve(smem_raw, p.C);
   const int warp = threadIdx.x >> 5;
+  if (threadIdx.x == 32 && p.paged) {
+    // The page-table line of this CTA's first tile, were every length at its bound (exact
+    // for equal lengths; a mere extra prefetch otherwise), is brought into L2 meanwhile.
+    const int HR = p.hkv * p.row_blocks;
+    const long long ut = (p.len_bound + kTileKeys - 1) / kTileKeys + p.draft_tiles;
+    const long long T = static_cast<long long>(p.C) * HR * ut;
+    const long long t0 = static_cast<long long>(blockIdx.x) * ((T + p.num_ctas - 1) / p.num_ctas);
+    const long long c = t0 / (HR * ut), lt = (t0 - c * HR * ut) % ut;
+    const long long pg = lt * kTileKeys / p.page_size;
+    if (c < p.C && lt * kTileKeys < p.len_bound && pg < p.max_pages)
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(p.page_table + c * p.max_pages + pg));
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kNK; ++s) mbar_init(smem_addr(&sm.kfull[s]), 1);
     for (int s = 0; s < kNV; ++s) {
@@ -773,7 +788,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_relinquish();
   }
   tc_fence_before();
-  build_plan(p, sm.len, sm.base);  // block-wide barriers inside
+  build_plan(p, sm.len, sm.base, len0);  // block-wide barriers inside
   tc_fence_after();
   const uint32_t tmem = *sm.tmem_base;
   const Cursor cu = cursor_begin(p, sm.len, sm.base);

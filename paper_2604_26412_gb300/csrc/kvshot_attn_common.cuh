@@ -202,12 +202,22 @@ __device__ __forceinline__ int clamp_len(const AttnParams& p, int c) {
   return L;
 }
 
+// Clamped prefix length of cache c from its already loaded entry.
+__device__ __forceinline__ int clamp_len_of(const AttnParams& p, int L) {
+  if (L < 0 || L > p.len_bound) {
+    set_error(p.err, KVSHOT_ERR_DEVICE_BOUNDS);
+    L = L < 0 ? 0 : p.len_bound;
+  }
+  return L;
+}
+
 // s_len[c] = clamped L_c; s_base[c] = first global tile of cache c (prefix sum of
-// units x tiles per unit).  Whole block participates.
-__device__ __forceinline__ void build_plan(const AttnParams& p, int* s_len, int* s_base) {
+// units x tiles per unit).  Whole block participates.  `len0` may hold
+// seq_lens[threadIdx.x], loaded early by the caller (-1: not loaded).
+__device__ __forceinline__ void build_plan(const AttnParams& p, int* s_len, int* s_base, int len0 = -1) {
   const int HR = p.hkv * p.row_blocks;
   for (int c = threadIdx.x; c < p.C; c += blockDim.x) {
-    const int L = clamp_len(p, c);
+    const int L = (c == static_cast<int>(threadIdx.x) && len0 >= 0) ? clamp_len_of(p, len0) : clamp_len(p, c);
     s_len[c] = L;
     s_base[c + 1] = ((L + kTileKeys - 1) / kTileKeys + p.draft_tiles) * HR;
   }
