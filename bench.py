@@ -98,10 +98,15 @@ def measured_peaks():
         return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
 
 
+# Sources of the draft-attention call (the kernels whose DRAM traffic profiles/traffic.json records).
+ATTN_SOURCES = ("attn_cc.cu", "attn_mma.cu", "attn_tc.cu", "kvshot_api.cu", "kvshot_attn_common.cuh",
+                "kvshot_internal.h", "merge_append.cu")
+
+
 def kernel_source_hash():
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2604_26412_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
+    for name in ATTN_SOURCES:
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode() + f.read())
     return h.hexdigest()[:16]
