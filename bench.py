@@ -100,7 +100,7 @@ def measured_peaks():
 
 # Sources of the draft-attention call (the kernels whose DRAM traffic profiles/traffic.json records).
 ATTN_SOURCES = ("attn_cc.cu", "attn_mma.cu", "attn_tc.cu", "kvshot_api.cu", "kvshot_attn_common.cuh",
-                "kvshot_internal.h", "merge_append.cu")
+                "kvshot_internal.h", "kvshot_tcgen05.cuh", "merge_append.cu")
 
 
 def kernel_source_hash():

@@ -187,6 +187,46 @@ kvshot_status kvshot_draft_append(const kvshot_attn_desc* desc, const void* q_in
                                   float rope_base, void* draft_k, void* draft_v, void* q_out,
                                   kvshot_stream_t stream);
 
+/*
+ * Gated-delta fusion of the hybrid drafter (Sec. 3.4, Eqs. "self-attn",
+ * "cross-attn", "delta" and "fusion").  For every draft token t, with n_t the
+ * self-attention branch (the EAGLE-3 path) and o_t the cross-attention
+ * branch (re-attention to the target KV):
+ *   delta_t = o_t - n_t
+ *   g_t     = sigmoid(W_g [n_t; o_t; delta_t] + b_g)
+ *   h_t     = n_t + g_t (.) (W_delta delta_t)
+ * The attention of both branches is kvshot_draft_attn: over the target prefix
+ * and the draft KV for o, over the drafter's own draft KV alone (every
+ * seq_lens[c] = 0) for n.  Products accumulate in fp32 and delta is never
+ * rounded (W delta is formed as W o - W n in fp32); h is rounded once to bf16
+ * (nearest even).
+ *
+ * n, o:     [T, d] bf16, row-major (token-major), 16-byte aligned.
+ * w_g:      [d, 3d] bf16, row-major: row i holds output feature i's weights
+ *           over the inputs [n; o; delta].  16-byte aligned.
+ * b_g:      [d] bf16, 8-byte aligned.
+ * w_delta:  [d, d] bf16, row-major, 16-byte aligned.
+ * h:        [T, d] bf16, 8-byte aligned; must not overlap n, o or the workspace.
+ * desc->hidden = d: a positive multiple of 128, at most 32768 (else
+ * KVSHOT_ERR_UNSUPPORTED); desc->num_tokens = T >= 0 (0: no-op), T * d < 2^31.
+ * Workspace: kvshot_gated_delta_workspace_size(desc) bytes (the fp32 partial
+ * products, 16 T d bytes), 256-byte aligned; nothing in it has to be
+ * initialised.  Errors follow the conventions at the top of this file.
+ */
+typedef struct kvshot_fusion_desc {
+  int32_t num_tokens;        /* T */
+  int32_t hidden;            /* d */
+  void* workspace;           /* device scratch, 256-byte aligned */
+  size_t workspace_bytes;
+  int32_t* err_flag;         /* optional device int32, 0 before the call (KVSHOT_ERR_TIMEOUT) */
+} kvshot_fusion_desc;
+
+/* Bytes of workspace kvshot_gated_delta needs; 0 if the descriptor is invalid. */
+size_t kvshot_gated_delta_workspace_size(const kvshot_fusion_desc* desc);
+
+kvshot_status kvshot_gated_delta(const kvshot_fusion_desc* desc, const void* n, const void* o, const void* w_g,
+                                 const void* b_g, const void* w_delta, void* h, kvshot_stream_t stream);
+
 /* Static description of a status code (never NULL). */
 const char* kvshot_status_string(kvshot_status status);
 

@@ -19,7 +19,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libkvshot.so")
-SOURCES = ["kvshot_api.cu", "attn_cc.cu", "attn_mma.cu", "merge_append.cu", "kvshot_static_ws.cu", "attn_tc.cu"]
+SOURCES = ["kvshot_api.cu", "attn_cc.cu", "attn_mma.cu", "merge_append.cu", "kvshot_static_ws.cu", "attn_tc.cu",
+           "gated_delta.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 _lock = threading.Lock()
 

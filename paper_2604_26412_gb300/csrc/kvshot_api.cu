@@ -55,6 +55,23 @@ bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box
 
 enum class Kernel { kCudaCore, kMma, kTensorMemory };
 
+}  // namespace
+
+bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_cols,
+                    uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
+  const cuuint32_t box[2] = {box_cols, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+namespace {
+
 // 4-D view {128 dims, hq, Nq, C} of q [C, Nq, hq, 128]; a box is one 64-dim
 // half of `heads` heads of one KV group for `nodes` draft nodes (rows node-major).
 bool encode_q(CUtensorMap* map, const void* q, int C, int Nq, int hq, QBox qb) {

@@ -88,6 +88,12 @@ struct TensorMaps {
   CUtensorMap q;  // [C, Nq, hq, 128] as 4-D {128, hq, Nq, C}; used by the tensor-memory kernel
 };
 
+// Encodes a 2-D tiled tensor map over a row-major bf16 matrix [rows, cols] (row pitch cols * 2
+// bytes), boxes of {box_cols, box_rows}, 128-byte swizzle.  False if the encoder is unavailable
+// or rejects the layout.
+bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_cols,
+                    uint32_t box_rows);
+
 // Kernel launchers (one per translation unit).  Return cudaSuccess or the launch error.
 cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, cudaStream_t stream);
 cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, cudaStream_t stream);

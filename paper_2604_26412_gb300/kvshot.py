@@ -1,7 +1,7 @@
 """Thin Python binding of libkvshot's C ABI (include/kvshot.h).
 
-Argument marshalling only: every step of draft attention and draft append
-runs in the library's CUDA kernels.  Tensors are torch CUDA tensors (or raw
+Argument marshalling only: every step of draft attention, draft append and
+the gated-delta fusion runs in the library's CUDA kernels.  Tensors are torch CUDA tensors (or raw
 device pointers as ints); the current torch stream is used unless a stream
 is given.  If the shared library is missing this module raises on import of
 the library -- there is no CPU fallback.
@@ -33,7 +33,7 @@ KVSHOT_FORCE_MMA = 0x4
 KVSHOT_FORCE_TC = 0x8
 
 EXPORTS = ("kvshot_draft_attn", "kvshot_draft_attn_workspace_size", "kvshot_draft_append", "kvshot_status_string",
-           "kvshot_version", "kvshot_draft_attn_static")
+           "kvshot_version", "kvshot_draft_attn_static", "kvshot_gated_delta", "kvshot_gated_delta_workspace_size")
 STATIC_WORKSPACE_BYTES = 32 * 1024 * 1024  # KVSHOT_STATIC_WORKSPACE_BYTES
 
 
@@ -69,6 +69,18 @@ class AttnDesc(ctypes.Structure):
     ]
 
 
+class FusionDesc(ctypes.Structure):
+    """Mirror of kvshot_fusion_desc."""
+
+    _fields_ = [
+        ("num_tokens", ctypes.c_int32),
+        ("hidden", ctypes.c_int32),
+        ("workspace", ctypes.c_void_p),
+        ("workspace_bytes", ctypes.c_size_t),
+        ("err_flag", ctypes.c_void_p),
+    ]
+
+
 _lib = None
 
 
@@ -97,6 +109,10 @@ def load(build_if_missing: bool = True):
     lib.kvshot_draft_append.argtypes = [ctypes.POINTER(AttnDesc), P, P, P, P, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_float, P, P, P, P]
     lib.kvshot_draft_append.restype = ctypes.c_int
+    lib.kvshot_gated_delta.argtypes = [ctypes.POINTER(FusionDesc), P, P, P, P, P, P, P]
+    lib.kvshot_gated_delta.restype = ctypes.c_int
+    lib.kvshot_gated_delta_workspace_size.argtypes = [ctypes.POINTER(FusionDesc)]
+    lib.kvshot_gated_delta_workspace_size.restype = ctypes.c_size_t
     lib.kvshot_status_string.argtypes = [ctypes.c_int]
     lib.kvshot_status_string.restype = ctypes.c_char_p
     lib.kvshot_version.argtypes = []
@@ -184,3 +200,23 @@ def draft_append(desc: AttnDesc, q_in, k_in, v_in, positions, n0: int, n_new: in
     st = draft_append_status(desc, q_in, k_in, v_in, positions, n0, n_new, rope_base, draft_k, draft_v, q_out, stream)
     if st != KVSHOT_OK:
         raise KvshotError(st, "kvshot_draft_append")
+
+
+def make_fusion_desc(*, num_tokens, hidden, workspace=None, workspace_bytes=0, err_flag=None) -> FusionDesc:
+    return FusionDesc(int(num_tokens), int(hidden), _ptr(workspace), int(workspace_bytes), _ptr(err_flag))
+
+
+def gated_delta_workspace_size(desc: FusionDesc) -> int:
+    return int(load().kvshot_gated_delta_workspace_size(_dref(desc)))
+
+
+def gated_delta_status(desc: FusionDesc, n, o, w_g, b_g, w_delta, h, stream=None) -> int:
+    """Call kvshot_gated_delta (h = n + sigmoid(W_g [n; o; o - n] + b_g) * W_delta (o - n)); return its status."""
+    return int(load().kvshot_gated_delta(_dref(desc), _ptr(n), _ptr(o), _ptr(w_g), _ptr(b_g), _ptr(w_delta),
+                                         _ptr(h), _stream(stream)))
+
+
+def gated_delta(desc: FusionDesc, n, o, w_g, b_g, w_delta, h, stream=None) -> None:
+    st = gated_delta_status(desc, n, o, w_g, b_g, w_delta, h, stream)
+    if st != KVSHOT_OK:
+        raise KvshotError(st, "kvshot_gated_delta")

@@ -249,3 +249,29 @@ def bf16_bits(t: torch.Tensor) -> np.ndarray:
 
 def bits_to_bf16(a: np.ndarray) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+
+
+HIDDEN = HQ * HEAD_DIM  # d of the hybrid drafter (Qwen3-8B hidden size; the two branches' width)
+
+
+@dataclasses.dataclass
+class FusionInputs:
+    """Inputs of the gated-delta fusion: the branches n, o [T, d] and the fusion weights (bf16)."""
+    n: torch.Tensor
+    o: torch.Tensor
+    w_g: torch.Tensor       # [d, 3d]
+    b_g: torch.Tensor       # [d]
+    w_delta: torch.Tensor   # [d, d]
+
+
+def fusion_inputs(T: int, d: int = HIDDEN, device="cpu", seed: int = 5) -> FusionInputs:
+    """Seeded stand-ins for the hybrid drafter's fusion step (Sec. 3.4): the two attention branches
+    ~N(0, 1) (attention outputs of unit-variance values), W_g ~N(0, 1/(3d)) and W_delta ~N(0, 1/d)
+    so the gate's pre-activation and the projected correction stay O(1), b_g ~N(0, 0.1^2).  No trained
+    weights exist here; these only fix shapes and scales."""
+    g = torch.Generator().manual_seed(seed)
+    t = dict(n=_randn_bf16((T, d), g, "cpu"), o=_randn_bf16((T, d), g, "cpu"),
+             w_g=_randn_bf16((d, 3 * d), g, "cpu", std=1.0 / math.sqrt(3 * d)),
+             b_g=_randn_bf16((d,), g, "cpu", std=0.1),
+             w_delta=_randn_bf16((d, d), g, "cpu", std=1.0 / math.sqrt(d)))
+    return FusionInputs(**{k: v.to(device) for k, v in t.items()})

@@ -139,3 +139,48 @@ def test_append_argument_codes(lib):
     assert call(qo=A + 256) == kvshot.KVSHOT_ERR_SHAPE                 # partial overlap of q_out and q_in
     assert kvshot.draft_append_status(_desc(head_dim=96), A, A, A, A, 0, 1, 1e6, A, A, A, stream=0) == \
         kvshot.KVSHOT_ERR_UNSUPPORTED
+
+
+def test_fusion_descriptor_layout_matches_header(tmp_path):
+    fields = [f for f, _ in kvshot.FusionDesc._fields_]
+    src = ["#include <stdio.h>", "#include <stddef.h>", '#include "kvshot.h"', "int main(void) {",
+           'printf("%zu\\n", sizeof(kvshot_fusion_desc));']
+    src += [f'printf("%zu\\n", offsetof(kvshot_fusion_desc, {f}));' for f in fields]
+    src += ["return 0; }"]
+    c = tmp_path / "layout_fusion.c"
+    c.write_text("\n".join(src))
+    exe = tmp_path / "layout_fusion"
+    subprocess.run(["gcc", "-I", os.path.dirname(HEADER), str(c), "-o", str(exe)], check=True)
+    vals = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    assert vals[0] == ctypes.sizeof(kvshot.FusionDesc)
+    for f, off in zip(fields, vals[1:]):
+        assert getattr(kvshot.FusionDesc, f).offset == off, f
+
+
+def test_fusion_argument_codes(lib):
+    """Every case fails validation (or is the T = 0 no-op) before anything is launched."""
+    T, D = 4, 256
+    ws = 16 * T * D
+
+    def call(desc, **k):
+        return kvshot.gated_delta_status(desc, k.get("n", A), k.get("o", A), k.get("wg", 2 * A), k.get("bg", 3 * A),
+                                         k.get("wd", 4 * A), k.get("h", 5 * A), stream=0)
+
+    good = kvshot.make_fusion_desc(num_tokens=T, hidden=D, workspace=6 * A, workspace_bytes=ws)
+    assert kvshot.gated_delta_workspace_size(good) == ws
+    assert call(None) == kvshot.KVSHOT_ERR_NULL
+    assert call(kvshot.make_fusion_desc(num_tokens=-1, hidden=D)) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(kvshot.make_fusion_desc(num_tokens=T, hidden=0)) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(kvshot.make_fusion_desc(num_tokens=T, hidden=200)) == kvshot.KVSHOT_ERR_UNSUPPORTED
+    assert call(kvshot.make_fusion_desc(num_tokens=T, hidden=65536)) == kvshot.KVSHOT_ERR_UNSUPPORTED
+    assert kvshot.gated_delta_workspace_size(kvshot.make_fusion_desc(num_tokens=T, hidden=200)) == 0
+    assert call(good, n=None) == kvshot.KVSHOT_ERR_NULL
+    assert call(good, wd=None) == kvshot.KVSHOT_ERR_NULL
+    assert call(good, n=A + 8) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(good, wg=2 * A + 4) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(good, h=5 * A + 2) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(kvshot.make_fusion_desc(num_tokens=T, hidden=D, workspace=6 * A, workspace_bytes=ws - 1)) == \
+        kvshot.KVSHOT_ERR_WORKSPACE
+    assert call(kvshot.make_fusion_desc(num_tokens=T, hidden=D, workspace=6 * A + 16, workspace_bytes=ws)) == \
+        kvshot.KVSHOT_ERR_WORKSPACE
+    assert call(kvshot.make_fusion_desc(num_tokens=0, hidden=D)) == kvshot.KVSHOT_OK  # no-op
