@@ -51,6 +51,9 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--part", choices=["attn", "fusion"], default="attn",
+                    help="attn: the draft-attention step (default); fusion: the hybrid drafter's gated-delta "
+                         "fusion at the hybrid-tree workload's per-depth token counts")
     ap.add_argument("--workload", type=int, default=5, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--mode", choices=["per_depth", "whole"], default="per_depth")
     ap.add_argument("--kernel", choices=["auto", "cc", "mma", "tc"], default="auto")
@@ -420,6 +423,177 @@ def run_ours(args, world, rank, local):
     return result
 
 
+FUSION_METRIC = "gated-delta fusion tokens/s and achieved HBM GB/s (fraction of GB300 peak) at 1 GPU"
+
+
+def fusion_bytes(T: int, d: int) -> int:
+    """Algorithmic bytes of one fusion call: W_g and W_delta (4 d^2 bf16), b_g, n, o and h."""
+    return 2 * (4 * d * d + d + 3 * T * d)
+
+
+class FusionOracleSample:
+    """The fusion oracle (as it stands) on one level's tokens."""
+
+    def __init__(self, fi, T):
+        from oracle import fusion as fo
+        self.fo = fo
+        self.T = T
+        self.args = [wl.bf16_bits(x.cpu()) for x in (fi.n[:T], fi.o[:T], fi.w_g, fi.b_g, fi.w_delta)]
+        self.cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+
+    def timed(self, budget_s: float):
+        t0, calls = time.perf_counter(), 0
+        while True:
+            self.fo.gated_delta(*self.args)
+            calls += 1
+            if time.perf_counter() - t0 >= budget_s:
+                break
+        dt = time.perf_counter() - t0
+        return self.T * calls / dt, f"{calls} fusion calls of {self.T} tokens x d={self.args[0].shape[1]}, fp64 " \
+            f"oracle (numpy matrix products), {dt:.1f} s", dt
+
+
+def run_fusion(args, world, rank, local):
+    """The hybrid drafter's gated-delta fusion (Sec. 3.4) for the hybrid-tree workload: one call per
+    drafting depth on the tokens of that depth (sequences x level size), hidden size d = 4096."""
+    from paper_2604_26412_gb300 import kvshot
+    spec = wl.config(3, seed=args.seed)
+    d = wl.HIDDEN
+    tokens = [spec.num_seqs * lv for lv in spec.levels]
+    T_max = max(tokens)
+    fi = wl.fusion_inputs(T_max, d, device="cuda", seed=args.seed + 5)
+    stream = torch.cuda.Stream()
+    descs, outs = [], []
+    ws_bytes = max(kvshot.gated_delta_workspace_size(kvshot.make_fusion_desc(num_tokens=T, hidden=d)) for T in tokens)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for T in tokens:
+        descs.append(kvshot.make_fusion_desc(num_tokens=T, hidden=d, workspace=ws, workspace_bytes=ws_bytes,
+                                             err_flag=err))
+        outs.append(torch.empty((T, d), dtype=torch.bfloat16, device="cuda"))
+
+    def step():
+        for i, T in enumerate(tokens):
+            kvshot.gated_delta(descs[i], fi.n[:T], fi.o[:T], fi.w_g, fi.b_g, fi.w_delta, outs[i], stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            step()
+    torch.cuda.synchronize()
+    graph = None
+    if not args.no_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            step()
+        torch.cuda.synchronize()
+    run = (lambda: graph.replay()) if graph is not None else step
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(args.steps):
+            run()
+        t1.record(stream)
+    torch.cuda.synchronize()
+    clock_info = clocks.stop()
+    barrier(world)
+    ms_total = max_over_ranks(t0.elapsed_time(t1), world)
+    ms_per_step = ms_total / args.steps
+    value = replicas.whole_job_rate(sum(tokens), args.steps, world, ms_total)
+    assert int(err.item()) == 0, f"device error {int(err.item())}"
+
+    # live roofline: CUDA events around every call on the launching stream
+    reps = 30
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in tokens]
+          for _ in range(reps)]
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(2e7))
+        for r in range(reps):
+            for i, T in enumerate(tokens):
+                ev[r][i][0].record(stream)
+                kvshot.gated_delta(descs[i], fi.n[:T], fi.o[:T], fi.w_g, fi.b_g, fi.w_delta, outs[i], stream)
+                ev[r][i][1].record(stream)
+    torch.cuda.synchronize()
+    call_ms = [statistics.mean(ev[r][i][0].elapsed_time(ev[r][i][1]) for r in range(reps)) for i in range(len(tokens))]
+    call_bytes = [fusion_bytes(T, d) for T in tokens]
+    call_flops = [8 * T * d * d for T in tokens]
+    achieved = sum(call_bytes) / (sum(call_ms) / 1e3) / 1e9
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    roofline = {
+        "bound": "hbm",
+        "kernel": "kvshot_gated_delta (tcgen05 GEMM + gate kernels)",
+        "achieved": round(achieved, 1),
+        "peak": hbm_peak,
+        "unit": "GB/s",
+        "frac": round(achieved / hbm_peak, 4),
+        "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6.8 TB/s",
+        "traffic": None,
+        "algorithmic_bytes_per_call": int(statistics.mean(call_bytes)),
+        "call_us": round(statistics.mean(call_ms) * 1e3, 2),
+        "per_level_us": [round(x * 1e3, 2) for x in call_ms],
+        "achieved_tflops": round(sum(call_flops) / (sum(call_ms) / 1e3) / 1e12, 2),
+    }
+
+    # end to end: the branches copied in from pinned host memory and h copied back every step
+    n_h = fi.n.cpu().pin_memory()
+    o_h = fi.o.cpu().pin_memory()
+    h_h = [torch.empty((T, d), dtype=torch.bfloat16).pin_memory() for T in tokens]
+    n_d, o_d = torch.empty_like(fi.n), torch.empty_like(fi.o)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2e_steps = max(3, min(args.steps, 50))
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(e2e_steps):
+            n_d.copy_(n_h, non_blocking=True)
+            o_d.copy_(o_h, non_blocking=True)
+            for i, T in enumerate(tokens):
+                kvshot.gated_delta(descs[i], n_d[:T], o_d[:T], fi.w_g, fi.b_g, fi.w_delta, outs[i], stream)
+                h_h[i].copy_(outs[i], non_blocking=True)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+    e2e = {"value": round(replicas.whole_job_rate(sum(tokens), e2e_steps, world, e2e_ms), 1), "unit": UNIT,
+           "h2d_bytes_per_step": 2 * T_max * d * 2, "d2h_bytes_per_step": sum(tokens) * d * 2}
+
+    result = {
+        "metric": FUSION_METRIC,
+        "value": round(value, 1),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) branches, N(0,1/(3d)) W_g, N(0,1/d) W_delta; no trained weights)",
+        "config": {
+            "workload": "hybrid tree, gated-delta fusion step (Sec. 3.4)",
+            "hidden": d,
+            "tokens_per_call": tokens,
+            "tokens_per_step": sum(tokens),
+            "cuda_graph": graph is not None,
+            "l2": "weights (134 MB per call) larger than L2 (no flush)",
+            "parallelism": f"replicas x{world}",
+        },
+        "roofline": roofline,
+        "e2e": e2e,
+        "clocks": clock_info,
+        "gpu_launches": 2 * len(tokens) * args.steps,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        samp = FusionOracleSample(fi, tokens[len(tokens) // 2])
+        v, desc, _ = samp.timed(args.cpu_sample_seconds)
+        result["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": samp.cores, "kind": "oracle",
+                                  "sample": desc}
+    return result
+
+
 def run_e2e(args, step, inp, stream, world):
     """Same steps through the C ABI, with the per-step inputs copied from pinned
     host buffers and the outputs copied back inside the timed region."""
@@ -458,9 +632,38 @@ def run_e2e(args, step, inp, stream, world):
 
 # --------------------------------------------------------- reference arm
 
+def run_reference_fusion(args):
+    """The fusion oracle as it stands on the host cores; each step is one call on the tokens of the
+    hybrid-tree workload's widest drafting depth (d = 4096)."""
+    spec = wl.config(3, seed=args.seed)
+    T = spec.num_seqs * max(spec.levels)
+    samp = FusionOracleSample(wl.fusion_inputs(T, wl.HIDDEN, device="cpu", seed=args.seed + 5), T)
+    for _ in range(args.warmup):
+        samp.fo.gated_delta(*samp.args)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        samp.fo.gated_delta(*samp.args)
+    dt = time.perf_counter() - t0
+    value = T * args.steps / dt
+    return {
+        "impl": "reference", "metric": FUSION_METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; same shapes as the GPU arm)",
+        "config": {"workload": "hybrid tree, gated-delta fusion step (Sec. 3.4)", "hidden": wl.HIDDEN,
+                   "tokens_per_call": T, "parallelism": "host cores"},
+        "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": samp.cores, "kind": "oracle",
+                         "sample": f"{args.steps} fusion calls of {T} tokens, fp64 oracle"},
+        "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+
+
 def run_reference(args):
     """The CPU fp64 oracle as it stands, timed on the host cores; each step is
     one drafting level (append + attention) of one sequence of the workload."""
+    if args.part == "fusion":
+        return run_reference_fusion(args)
     spec = wl.config(args.workload, seed=args.seed)
     samp = OracleSample(spec, args.mode, args.seed)
     for w in range(args.warmup):
@@ -504,7 +707,7 @@ def main():
         print(json.dumps(run_reference(args)), flush=True)
         return
     world, rank, local = dist_setup()
-    result = run_ours(args, world, rank, local)
+    result = (run_fusion if args.part == "fusion" else run_ours)(args, world, rank, local)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:

@@ -40,7 +40,7 @@ using namespace tc;
 constexpr int kFeat = 128;                    // output features per CTA (MMA M)
 constexpr int kTok = 128;                     // tokens per CTA (MMA N per operand)
 constexpr int kKT = 64;                       // K per stage: one 128-byte swizzled row
-constexpr int kGemmStages = 4;
+constexpr int kGemmStages = 6;                // ring slots: blocks 0/1 use all 6 (32 KB each), blocks 2/3 four (48 KB)
 constexpr int kGemmThreads = 128;             // warp 0 lane 0: TMA; warp 1: TMEM owner, lane 0 MMA; all: epilogue
 constexpr int kABytes = kFeat * kKT * 2;      // 16 KB
 constexpr int kBBytes = 2 * kTok * kKT * 2;   // 32 KB: n rows then o rows
@@ -74,7 +74,9 @@ struct FusionMaps {
   CUtensorMap o;   // o [T, d], boxes {64, box_tok}
 };
 
-size_t gemm_smem_bytes() { return 1024 + kGemmStages * (kABytes + kBBytes) + 8 * (2 * kGemmStages + 1) + 16; }
+constexpr int kRingBytes = 4 * (kABytes + kBBytes);  // 192 KB: 6 x (A + one token tile) or 4 x (A + two)
+
+size_t gemm_smem_bytes() { return 1024 + kRingBytes + 8 * (2 * kGemmStages + 1) + 16; }
 
 // Grid (token blocks, feature blocks, 4 weight blocks).
 __global__ void __launch_bounds__(kGemmThreads, 1)
@@ -85,9 +87,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   const bool both = blk >= 2;  // B holds the n rows and the o rows
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sa = base;                                   // [stages][kABytes]
-  uint8_t* sb = sa + kGemmStages * kABytes;             // [stages][kBBytes]
-  uint64_t* full = reinterpret_cast<uint64_t*>(sb + kGemmStages * kBBytes);
+  // Ring slot s: A at base + s * slot, B right after it (one or two token tiles).
+  const int nst = both ? 4 : 6;
+  const int slot = kABytes + (both ? 2 : 1) * kTok * 128;
+  uint64_t* full = reinterpret_cast<uint64_t*>(base + kRingBytes);
   uint64_t* empty = full + kGemmStages;
   uint64_t* done = empty + kGemmStages;
   uint32_t* tmem_base = reinterpret_cast<uint32_t*>(done + 1);
@@ -118,13 +121,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int wx0 = blk == 3 ? 0 : blk * p.d;
     const uint32_t tx = kABytes + (both ? 2 : 1) * p.box_tok * 128;
     for (int kt = 0; kt < nk && ok; ++kt) {
-      const int s = kt % kGemmStages;
-      if (kt >= kGemmStages) ok = mbar_wait(smem_addr(&empty[s]), ((kt - kGemmStages) / kGemmStages) & 1, p.err);
+      const int s = kt % nst;
+      if (kt >= nst) ok = mbar_wait(smem_addr(&empty[s]), ((kt - nst) / nst) & 1, p.err);
       if (!ok) break;
       const uint32_t fb = smem_addr(&full[s]);
       mbar_arrive_expect_tx(fb, tx);
-      tma_load_2d(smem_addr(sa + s * kABytes), wmap, wx0 + kt * kKT, ft * kFeat, fb, stream_once);
-      const uint32_t bdst = smem_addr(sb + s * kBBytes);
+      tma_load_2d(smem_addr(base + s * slot), wmap, wx0 + kt * kKT, ft * kFeat, fb, stream_once);
+      const uint32_t bdst = smem_addr(base + s * slot + kABytes);
       const int ty = tt * kTok;
       if (blk == 1) {
         tma_load_2d_nohint(bdst, &maps.o, kt * kKT, ty, fb);
@@ -136,11 +139,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   } else if (warp == 1 && lane == 0) {
     const uint32_t idesc = idesc_bf16(kFeat, both ? 2 * kTok : kTok, false);
     for (int kt = 0; kt < nk && ok; ++kt) {
-      const int s = kt % kGemmStages;
-      ok = mbar_wait(smem_addr(&full[s]), (kt / kGemmStages) & 1, p.err);
+      const int s = kt % nst;
+      ok = mbar_wait(smem_addr(&full[s]), (kt / nst) & 1, p.err);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t a0 = smem_addr(sa + s * kABytes), b0 = smem_addr(sb + s * kBBytes);
+      const uint32_t a0 = smem_addr(base + s * slot), b0 = a0 + kABytes;
 #pragma unroll
       for (int ks = 0; ks < kKT / 16; ++ks) {
         const uint64_t a = smem_desc_sw128(a0 + ks * 32, 16, 1024);
