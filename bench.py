@@ -106,25 +106,29 @@ ATTN_SOURCES = ("attn_cc.cu", "attn_mma.cu", "attn_tc.cu", "kvshot_api.cu", "kvs
                 "kvshot_internal.h", "kvshot_tcgen05.cuh", "merge_append.cu")
 
 
-def kernel_source_hash():
+# Sources of the gated-delta fusion call.
+FUSION_SOURCES = ("gated_delta.cu", "kvshot_attn_common.cuh", "kvshot_internal.h", "kvshot_tcgen05.cuh")
+
+
+def kernel_source_hash(sources=ATTN_SOURCES):
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2604_26412_gb300", "csrc")
-    for name in ATTN_SOURCES:
+    for name in sources:
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode() + f.read())
     return h.hexdigest()[:16]
 
 
 def recorded_traffic(workload, mode, kernel_hash):
-    """DRAM bytes per draft-attention call from a committed ncu summary, if it is
-    for the current kernel sources; else None."""
+    """DRAM bytes per call (key "w<workload>-<mode>", or "fusion-hybrid_tree") from a committed ncu
+    summary, if it is for the current kernel sources; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)
     except (OSError, ValueError):
         return None
-    key = f"w{workload}-{mode}"
+    key = f"w{workload}-{mode}" if workload is not None else mode
     e = rec.get(key)
     if not e or e.get("kernel_hash") != kernel_hash:
         return None
@@ -531,11 +535,12 @@ def run_fusion(args, world, rank, local):
         "unit": "GB/s",
         "frac": round(achieved / hbm_peak, 4),
         "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6.8 TB/s",
-        "traffic": None,
+        "traffic": recorded_traffic(None, "fusion-hybrid_tree", kernel_source_hash(FUSION_SOURCES)),
         "algorithmic_bytes_per_call": int(statistics.mean(call_bytes)),
         "call_us": round(statistics.mean(call_ms) * 1e3, 2),
         "per_level_us": [round(x * 1e3, 2) for x in call_ms],
         "achieved_tflops": round(sum(call_flops) / (sum(call_ms) / 1e3) / 1e12, 2),
+        "kernel_hash": kernel_source_hash(FUSION_SOURCES),
     }
 
     # end to end: the branches copied in from pinned host memory and h copied back every step
