@@ -61,6 +61,13 @@ typedef enum kvshot_status {
 #define KVSHOT_FORCE_CC 0x2u   /* use the CUDA-core kernel whatever the row count (measurement aid) */
 #define KVSHOT_FORCE_MMA 0x4u  /* use the mma.sync tensor-core kernel whatever the row count (measurement aid) */
 #define KVSHOT_FORCE_TC 0x8u   /* use the tcgen05 / tensor-memory kernel (needs 128 % (hq / hkv) == 0) */
+/* Let the attention kernel start while the kernel enqueued just before the call is still running
+ * (programmatic dependent launch): it then reads seq_lens, page_table, target_k/v and tree_parent,
+ * and starts the first target K/V loads, before that kernel has finished, and waits for it only
+ * before it reads q or draft_k/v or writes anything.  Set it only when the preceding kernel does
+ * not write seq_lens, page_table, target_k, target_v or tree_parent (kvshot_draft_append, which
+ * writes q and the draft K/V, qualifies). */
+#define KVSHOT_OVERLAP_PREVIOUS 0x10u
 
 /*
  * Problem descriptor shared by kvshot_draft_attn and kvshot_draft_append.

@@ -316,6 +316,9 @@ __global__ void __launch_bounds__(kThreads, 2)
     prefetch_tensormap(&maps.dv);
   }
   build_plan(p, sm.len, sm.base);  // contains __syncthreads
+  // With KVSHOT_OVERLAP_PREVIOUS the kernel may have started before the preceding kernel ended:
+  // q and the draft K/V (and every output) are touched only after it has.
+  wait_for_prerequisite_grid();
   const Cursor cu = cursor_begin(p, sm.len, sm.base);
   Pipe pipe{sm.ring, sm.full, sm.empty, kStages, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
   if (warp == kWarps) {
@@ -341,13 +344,12 @@ cudaError_t attn_cc_occupancy(int C, int* ctas_per_sm) {
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, attn_cc_kernel, kThreads, smem);
 }
 
-cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, cudaStream_t stream) {
+cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, bool pdl, cudaStream_t stream) {
   const size_t smem = smem_bytes(p.C);
   cudaError_t e = cudaFuncSetAttribute(attn_cc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  attn_cc_kernel<<<p.num_ctas, kThreads, smem, stream>>>(p, maps);
-  return cudaGetLastError();
+  return launch_maybe_pdl(attn_cc_kernel, dim3(p.num_ctas), dim3(kThreads), smem, pdl, stream, p, maps);
 }
 
 }  // namespace kvshot

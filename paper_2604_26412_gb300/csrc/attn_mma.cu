@@ -363,6 +363,9 @@ __global__ void __launch_bounds__(CF::kThreads, CF::kMinBlocks)
     prefetch_tensormap(&maps.dv);
   }
   build_plan(p, sm.len, sm.base);
+  // With KVSHOT_OVERLAP_PREVIOUS the kernel may have started before the preceding kernel ended:
+  // q and the draft K/V (and every output) are touched only after it has.
+  wait_for_prerequisite_grid();
   const Cursor cu = cursor_begin(p, sm.len, sm.base);
   Pipe pipe{sm.ring, sm.full, sm.empty, CF::kStages, reinterpret_cast<volatile int*>(&sm.misc[0]), &sm.misc[1]};
   if (warp == CF::kWarps) {
@@ -380,13 +383,12 @@ using Cfg3 = Cfg<3, 2, 4, 1>;
 using Cfg4 = Cfg<4, 2, 4, 1>;
 
 template <class CF>
-cudaError_t launch_cfg(const AttnParams& p, const TensorMaps& maps, cudaStream_t stream) {
+cudaError_t launch_cfg(const AttnParams& p, const TensorMaps& maps, bool pdl, cudaStream_t stream) {
   const size_t smem = smem_bytes<CF>(p.C);
   cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<CF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  attn_mma_kernel<CF><<<p.num_ctas, CF::kThreads, smem, stream>>>(p, maps);
-  return cudaGetLastError();
+  return launch_maybe_pdl(attn_mma_kernel<CF>, dim3(p.num_ctas), dim3(CF::kThreads), smem, pdl, stream, p, maps);
 }
 
 template <class CF>
@@ -412,12 +414,12 @@ cudaError_t attn_mma_occupancy(int m_tiles, int C, int* ctas_per_sm) {
   }
 }
 
-cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, cudaStream_t stream) {
+cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, bool pdl, cudaStream_t stream) {
   switch (m_tiles) {
-    case 1: return launch_cfg<Cfg1>(p, maps, stream);
-    case 2: return launch_cfg<Cfg2>(p, maps, stream);
-    case 3: return launch_cfg<Cfg3>(p, maps, stream);
-    case 4: return launch_cfg<Cfg4>(p, maps, stream);
+    case 1: return launch_cfg<Cfg1>(p, maps, pdl, stream);
+    case 2: return launch_cfg<Cfg2>(p, maps, pdl, stream);
+    case 3: return launch_cfg<Cfg3>(p, maps, pdl, stream);
+    case 4: return launch_cfg<Cfg4>(p, maps, pdl, stream);
     default: return cudaErrorInvalidValue;
   }
 }

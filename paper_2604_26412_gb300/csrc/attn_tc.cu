@@ -238,6 +238,9 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
   bool valid = false, warp_live = false;
   float m_run = -INFINITY, l_run = 0.f;  // l_run: this thread's columns only (spread)
   int t = 0, anc_seq = -1;
+  // Outputs and the workspace are written only once the preceding kernel has ended
+  // (KVSHOT_OVERLAP_PREVIOUS); the first S needs q, which comes after that anyway.
+  wait_for_prerequisite_grid();
   for (; cu.t < cu.t_end; cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
     if (cu.c != unit_c || cu.hr != unit_hr) {
@@ -538,6 +541,7 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
   const FastDiv pdiv(p.paged ? p.page_size : 1, small), rbdiv(p.row_blocks, true);
   int unit_c = -1, unit_hr = -1, h = 0, pages = 0;  // the current unit's KV head and its cache's pages
   int ok = 1;
+  bool waited = false;  // griddepcontrol.wait done
   for (; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
     const bool first = cu.t == cu.t_begin || cu.lt == 0;  // first tile of a piece
     const bool mine = (t & 1) == role;
@@ -552,6 +556,10 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
       pages = p.paged ? pdiv.div(cu.L + p.page_size - 1) : 0;
     }
     if (first && role == 1) {  // the unit's q block
+      if (!waited) {  // q may come from the preceding kernel (KVSHOT_OVERLAP_PREVIOUS)
+        wait_for_prerequisite_grid();
+        waited = true;
+      }
       if (lane == 0) {
         const uint32_t qbar = smem_addr(sm.qfull);
         ok = mbar_wait(smem_addr(sm.qempty), (piece & 1) ^ 1u, p.err) && !*pipe.abort;
@@ -580,6 +588,10 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
     piece += first;
     if (!mine) continue;
     const TileBoxes tb = tile_boxes(p, cu, win, lane, h, pages, pdiv);
+    if (tb.draft && !waited) {  // so may the draft K/V; the target K/V before them may not
+      wait_for_prerequisite_grid();
+      waited = true;
+    }
     // Lanes 0..15 load the K boxes, lanes 16..31 the V boxes (half = lane & 1, row group = (lane & 15) >> 1).
     const int kv = lane >> 4, hf = lane & 1, i = (lane & 15) >> 1;
     const uint32_t tx = tb.nbox * tb.br * 128 * 2;  // bytes of one K (or V) tile's boxes
@@ -716,13 +728,13 @@ cudaError_t attn_tc_occupancy(int C, int* ctas_per_sm) {
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, attn_tc_kernel<false>, kThreads, smem);
 }
 
-cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, cudaStream_t stream) {
+cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, bool pdl,
+                           cudaStream_t stream) {
   const size_t smem = smem_bytes(p.C);
   auto* kernel = spread ? attn_tc_kernel<true> : attn_tc_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  kernel<<<p.num_ctas, kThreads, smem, stream>>>(p, maps, nq_box);
-  return cudaGetLastError();
+  return launch_maybe_pdl(kernel, dim3(p.num_ctas), dim3(kThreads), smem, pdl, stream, p, maps, nq_box);
 }
 
 }  // namespace kvshot

@@ -124,7 +124,7 @@ kvshot_status check_common(const kvshot_attn_desc* d) {
   if (d->n_nodes < 0 || d->n_query < 0 || d->n_query > d->n_nodes || d->n_nodes > d->n_max) return KVSHOT_ERR_SHAPE;
   if (d->max_seq_len < 0) return KVSHOT_ERR_SHAPE;
   if (!std::isfinite(d->scale)) return KVSHOT_ERR_SHAPE;
-  const uint32_t known = KVSHOT_TREE | KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC;
+  const uint32_t known = KVSHOT_TREE | KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC | KVSHOT_OVERLAP_PREVIOUS;
   if ((d->flags & ~known) != 0) return KVSHOT_ERR_SHAPE;
   const uint32_t force = d->flags & (KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC);
   if (force & (force - 1)) return KVSHOT_ERR_SHAPE;  // at most one kernel may be forced
@@ -317,9 +317,10 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   p.num_ctas = pl.num_ctas;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  cudaError_t e = pl.kernel == Kernel::kMma            ? launch_attn_mma(p, maps, pl.m_tiles, s)
-                  : pl.kernel == Kernel::kTensorMemory ? launch_attn_tc(p, maps, pl.nq_box, pl.spread, s)
-                                                       : launch_attn_cc(p, maps, s);
+  const bool pdl = (d->flags & KVSHOT_OVERLAP_PREVIOUS) != 0;
+  cudaError_t e = pl.kernel == Kernel::kMma            ? launch_attn_mma(p, maps, pl.m_tiles, pdl, s)
+                  : pl.kernel == Kernel::kTensorMemory ? launch_attn_tc(p, maps, pl.nq_box, pl.spread, pdl, s)
+                                                       : launch_attn_cc(p, maps, pdl, s);
   if (e != cudaSuccess) return KVSHOT_ERR_CUDA;
   e = launch_merge(p, s);
   return e == cudaSuccess ? KVSHOT_OK : KVSHOT_ERR_CUDA;

@@ -94,10 +94,30 @@ struct TensorMaps {
 bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_cols,
                     uint32_t box_rows);
 
-// Kernel launchers (one per translation unit).  Return cudaSuccess or the launch error.
-cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, cudaStream_t stream);
-cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, cudaStream_t stream);
-cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, cudaStream_t stream);
+// Kernel launchers (one per translation unit).  Return cudaSuccess or the launch error.  `pdl`:
+// launch with programmatic stream serialization (KVSHOT_OVERLAP_PREVIOUS).
+cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, bool pdl, cudaStream_t stream);
+cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, bool pdl, cudaStream_t stream);
+cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, bool pdl,
+                           cudaStream_t stream);
+
+// Launches `kernel` on grid x block with `smem` dynamic bytes; with programmatic stream
+// serialization when `pdl` is set.
+template <typename... Args, typename... Actual>
+cudaError_t launch_maybe_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t smem, bool pdl,
+                             cudaStream_t stream, Actual&&... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Actual&&>(args)...);
+}
 cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream);
 cudaError_t launch_append(const AppendParams& a, cudaStream_t stream);
 

@@ -133,6 +133,8 @@ __device__ __forceinline__ __nv_bfloat16 rope_bf16(float a, float b, float c32, 
 // One CTA per (cache, new node).  Work item = (head, 16-byte chunk j0 of the
 // first half): it rotates dims j0..j0+7 together with their partners +64.
 __global__ void __launch_bounds__(kAppendThreads) append_kernel(const __grid_constant__ AppendParams a) {
+  // An attention call launched with KVSHOT_OVERLAP_PREVIOUS may start its prologue meanwhile.
+  if (threadIdx.x == 0) allow_dependent_launch();
   __shared__ double s_cos[kHeadDim / 2], s_sin[kHeadDim / 2];
   const int c = blockIdx.x / a.n_new, i = blockIdx.x - (blockIdx.x / a.n_new) * a.n_new;
   const int pos = a.positions[static_cast<size_t>(c) * a.n_new + i];

@@ -31,6 +31,7 @@ KVSHOT_TREE = 0x1
 KVSHOT_FORCE_CC = 0x2
 KVSHOT_FORCE_MMA = 0x4
 KVSHOT_FORCE_TC = 0x8
+KVSHOT_OVERLAP_PREVIOUS = 0x10
 
 EXPORTS = ("kvshot_draft_attn", "kvshot_draft_attn_workspace_size", "kvshot_draft_append", "kvshot_status_string",
            "kvshot_version", "kvshot_draft_attn_static", "kvshot_gated_delta", "kvshot_gated_delta_workspace_size")

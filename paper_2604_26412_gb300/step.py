@@ -56,8 +56,9 @@ class DraftStep:
                 n_max=inp.n_max, max_seq_len=s.max_seq_len, head_dim=s.head_dim,
                 page_size=s.page_size if paged else 0,
                 max_pages_per_seq=inp.page_table.shape[1] if paged else 0,
-                num_pages=inp.num_pages if paged else 0, l_cap=inp.l_cap, scale=scale, tree=s.tree, flags=flags,
-                num_ctas=num_ctas, err_flag=self.err))
+                num_pages=inp.num_pages if paged else 0, l_cap=inp.l_cap, scale=scale, tree=s.tree,
+                # the attention call follows this step's own append kernel, which writes only q and the draft K/V
+                flags=flags | kvshot.KVSHOT_OVERLAP_PREVIOUS, num_ctas=num_ctas, err_flag=self.err))
         ws = max(kvshot.workspace_size(d) for d in self.descs)
         if ws == 0:
             raise kvshot.KvshotError(kvshot.KVSHOT_ERR_SHAPE, "kvshot_draft_attn_workspace_size")

@@ -96,7 +96,7 @@ def _attn(d, **ptrs):
     (dict(num_pages=0), kvshot.KVSHOT_ERR_SHAPE),
     (dict(max_seq_len=-1), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=0x80), kvshot.KVSHOT_ERR_SHAPE),
-    (dict(flags=0x10), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(flags=0x20), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=kvshot.KVSHOT_FORCE_CC | kvshot.KVSHOT_FORCE_MMA), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=kvshot.KVSHOT_FORCE_MMA | kvshot.KVSHOT_FORCE_TC), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=kvshot.KVSHOT_FORCE_TC, hq=24, hkv=8), kvshot.KVSHOT_ERR_UNSUPPORTED),
