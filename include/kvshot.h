@@ -234,6 +234,59 @@ size_t kvshot_gated_delta_workspace_size(const kvshot_fusion_desc* desc);
 kvshot_status kvshot_gated_delta(const kvshot_fusion_desc* desc, const void* n, const void* o, const void* w_g,
                                  const void* b_g, const void* w_delta, void* h, kvshot_stream_t stream);
 
+/*
+ * Linear projection of multi-layer target KV for the KV-only drafter
+ * (Sec. 3.2, injection strategy "linear projection"; "Proj + RoPE fix").
+ * For every newly verified token t (desc->num_tokens = T of them), with
+ * d_kv = hkv * 128 and L = desc->num_layers sampled target layers:
+ *   K'(t) = W_K [K_1(t); ...; K_L(t)],   V'(t) = W_V [V_1(t); ...; V_L(t)]
+ * and, with KVSHOT_PROJECT_ROPE, K'(t) is rotated again by RoPE at the
+ * token's position (rotate-half pairs (j, j + 64) of every head,
+ * theta_j = pos * rope_base^(-2j/128), as in kvshot_draft_append).  K'(t) and
+ * V'(t) are rounded to bf16 and stored in slot positions[t] of cache
+ * token_cache[t] of the reused cache that kvshot_draft_attn reads as its
+ * target K/V; other slots are left untouched.  Products accumulate in fp32.
+ *
+ * k_in, v_in:  [T, L, hkv, 128] bf16: the tokens' K / V of the L layers (K post-RoPE, as cached).
+ * w_k, w_v:    [d_kv, L * d_kv] bf16, row-major (row i: output feature i over the concatenated inputs).
+ * token_cache: [T] int32 in [0, num_caches); positions: [T] int32 >= 0, below the cache's capacity.
+ * page_table:  paged cache (non-NULL): [num_caches, max_pages_per_seq] int32; k_out / v_out are
+ *              [num_pages, hkv, page_size, 128] bf16.  Contiguous (NULL): k_out / v_out are
+ *              [num_caches, hkv, l_cap, 128] bf16.
+ * All bf16 pointers 16-byte aligned, int32 pointers 4-byte aligned.  num_layers <= 8, hkv <= 64.
+ * Device-side errors (a cache, position or page id out of range) skip that token's store and set
+ * KVSHOT_ERR_DEVICE_BOUNDS.  T == 0 is a no-op.
+ * Workspace: kvshot_kv_project_workspace_size(desc) bytes (fp32 partial products), 256-byte aligned,
+ * no initialisation needed.
+ */
+#define KVSHOT_PROJECT_ROPE 0x1u /* re-apply RoPE to the projected keys ("Proj + RoPE fix") */
+
+typedef struct kvshot_project_desc {
+  int32_t num_tokens;        /* T */
+  int32_t num_layers;        /* L >= 1 */
+  int32_t hkv;               /* KV heads */
+  int32_t head_dim;          /* must be 128 */
+  int32_t num_caches;        /* caches of the output (reused) cache */
+  int32_t page_size;         /* paged output: tokens per page */
+  int32_t max_pages_per_seq; /* paged output: row stride of page_table */
+  int32_t num_pages;         /* paged output: pages in the pools */
+  int32_t l_cap;             /* contiguous output: token capacity per (cache, KV head) */
+  float rope_base;           /* > 0 (used with KVSHOT_PROJECT_ROPE) */
+  uint32_t flags;            /* KVSHOT_PROJECT_ROPE or 0 */
+  void* workspace;           /* device scratch, 256-byte aligned */
+  size_t workspace_bytes;
+  int32_t* err_flag;         /* optional device int32, 0 before the call */
+} kvshot_project_desc;
+
+/* Bytes of workspace kvshot_kv_project needs (0 if the descriptor is invalid; the layout is read
+ * from page_size > 0 for this query). */
+size_t kvshot_kv_project_workspace_size(const kvshot_project_desc* desc);
+
+kvshot_status kvshot_kv_project(const kvshot_project_desc* desc, const void* k_in, const void* v_in,
+                                const void* w_k, const void* w_v, const int32_t* token_cache,
+                                const int32_t* positions, const int32_t* page_table, void* k_out, void* v_out,
+                                kvshot_stream_t stream);
+
 /* Static description of a status code (never NULL). */
 const char* kvshot_status_string(kvshot_status status);
 

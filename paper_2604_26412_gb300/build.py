@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libkvshot.so")
 SOURCES = ["kvshot_api.cu", "attn_cc.cu", "attn_mma.cu", "merge_append.cu", "kvshot_static_ws.cu", "attn_tc.cu",
-           "gated_delta.cu"]
+           "gated_delta.cu", "kv_project.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 _lock = threading.Lock()
 

@@ -34,7 +34,9 @@ KVSHOT_FORCE_TC = 0x8
 KVSHOT_OVERLAP_PREVIOUS = 0x10
 
 EXPORTS = ("kvshot_draft_attn", "kvshot_draft_attn_workspace_size", "kvshot_draft_append", "kvshot_status_string",
-           "kvshot_version", "kvshot_draft_attn_static", "kvshot_gated_delta", "kvshot_gated_delta_workspace_size")
+           "kvshot_version", "kvshot_draft_attn_static", "kvshot_gated_delta", "kvshot_gated_delta_workspace_size",
+           "kvshot_kv_project", "kvshot_kv_project_workspace_size")
+KVSHOT_PROJECT_ROPE = 0x1
 STATIC_WORKSPACE_BYTES = 32 * 1024 * 1024  # KVSHOT_STATIC_WORKSPACE_BYTES
 
 
@@ -82,6 +84,27 @@ class FusionDesc(ctypes.Structure):
     ]
 
 
+class ProjectDesc(ctypes.Structure):
+    """Mirror of kvshot_project_desc."""
+
+    _fields_ = [
+        ("num_tokens", ctypes.c_int32),
+        ("num_layers", ctypes.c_int32),
+        ("hkv", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32),
+        ("num_caches", ctypes.c_int32),
+        ("page_size", ctypes.c_int32),
+        ("max_pages_per_seq", ctypes.c_int32),
+        ("num_pages", ctypes.c_int32),
+        ("l_cap", ctypes.c_int32),
+        ("rope_base", ctypes.c_float),
+        ("flags", ctypes.c_uint32),
+        ("workspace", ctypes.c_void_p),
+        ("workspace_bytes", ctypes.c_size_t),
+        ("err_flag", ctypes.c_void_p),
+    ]
+
+
 _lib = None
 
 
@@ -114,6 +137,10 @@ def load(build_if_missing: bool = True):
     lib.kvshot_gated_delta.restype = ctypes.c_int
     lib.kvshot_gated_delta_workspace_size.argtypes = [ctypes.POINTER(FusionDesc)]
     lib.kvshot_gated_delta_workspace_size.restype = ctypes.c_size_t
+    lib.kvshot_kv_project.argtypes = [ctypes.POINTER(ProjectDesc), P, P, P, P, P, P, P, P, P, P]
+    lib.kvshot_kv_project.restype = ctypes.c_int
+    lib.kvshot_kv_project_workspace_size.argtypes = [ctypes.POINTER(ProjectDesc)]
+    lib.kvshot_kv_project_workspace_size.restype = ctypes.c_size_t
     lib.kvshot_status_string.argtypes = [ctypes.c_int]
     lib.kvshot_status_string.restype = ctypes.c_char_p
     lib.kvshot_version.argtypes = []
@@ -221,3 +248,29 @@ def gated_delta(desc: FusionDesc, n, o, w_g, b_g, w_delta, h, stream=None) -> No
     st = gated_delta_status(desc, n, o, w_g, b_g, w_delta, h, stream)
     if st != KVSHOT_OK:
         raise KvshotError(st, "kvshot_gated_delta")
+
+
+def make_project_desc(*, num_tokens, num_layers, hkv, num_caches, head_dim=128, page_size=0, max_pages_per_seq=0,
+                      num_pages=0, l_cap=0, rope_base=1.0e6, rope=True, workspace=None, workspace_bytes=0,
+                      err_flag=None) -> ProjectDesc:
+    return ProjectDesc(int(num_tokens), int(num_layers), int(hkv), int(head_dim), int(num_caches), int(page_size),
+                       int(max_pages_per_seq), int(num_pages), int(l_cap), float(rope_base),
+                       KVSHOT_PROJECT_ROPE if rope else 0, _ptr(workspace), int(workspace_bytes), _ptr(err_flag))
+
+
+def kv_project_workspace_size(desc: ProjectDesc) -> int:
+    return int(load().kvshot_kv_project_workspace_size(_dref(desc)))
+
+
+def kv_project_status(desc: ProjectDesc, k_in, v_in, w_k, w_v, token_cache, positions, page_table, k_out, v_out,
+                      stream=None) -> int:
+    """Call kvshot_kv_project (K' = W_K [K_1..K_L] (+ RoPE), V' = W_V [V_1..V_L] into the reused cache)."""
+    return int(load().kvshot_kv_project(_dref(desc), _ptr(k_in), _ptr(v_in), _ptr(w_k), _ptr(w_v), _ptr(token_cache),
+                                        _ptr(positions), _ptr(page_table), _ptr(k_out), _ptr(v_out), _stream(stream)))
+
+
+def kv_project(desc: ProjectDesc, k_in, v_in, w_k, w_v, token_cache, positions, page_table, k_out, v_out,
+               stream=None) -> None:
+    st = kv_project_status(desc, k_in, v_in, w_k, w_v, token_cache, positions, page_table, k_out, v_out, stream)
+    if st != KVSHOT_OK:
+        raise KvshotError(st, "kvshot_kv_project")

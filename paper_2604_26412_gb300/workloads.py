@@ -275,3 +275,23 @@ def fusion_inputs(T: int, d: int = HIDDEN, device="cpu", seed: int = 5) -> Fusio
              b_g=_randn_bf16((d,), g, "cpu", std=0.1),
              w_delta=_randn_bf16((d, d), g, "cpu", std=1.0 / math.sqrt(d)))
     return FusionInputs(**{k: v.to(device) for k, v in t.items()})
+
+
+@dataclasses.dataclass
+class ProjectInputs:
+    """Inputs of the multi-layer KV projection: the new tokens' K/V of L layers and W_K, W_V (bf16)."""
+    k_in: torch.Tensor   # [T, L, hkv, 128]
+    v_in: torch.Tensor
+    w_k: torch.Tensor    # [hkv*128, L*hkv*128]
+    w_v: torch.Tensor
+
+
+def project_inputs(T: int, L: int = 3, hkv: int = HKV, device="cpu", seed: int = 7) -> ProjectInputs:
+    """Seeded stand-ins for the KV-only drafter's projection (Sec. 3.2): K/V ~N(0, 1) like the target
+    cache, W ~N(0, 1/(L d_kv)) so the projected vectors stay O(1).  L = 3 sampled layers (App. B)."""
+    g = torch.Generator().manual_seed(seed)
+    dkv = hkv * HEAD_DIM
+    t = dict(k_in=_randn_bf16((T, L, hkv, HEAD_DIM), g, "cpu"), v_in=_randn_bf16((T, L, hkv, HEAD_DIM), g, "cpu"),
+             w_k=_randn_bf16((dkv, L * dkv), g, "cpu", std=1.0 / math.sqrt(L * dkv)),
+             w_v=_randn_bf16((dkv, L * dkv), g, "cpu", std=1.0 / math.sqrt(L * dkv)))
+    return ProjectInputs(**{k: v.to(device) for k, v in t.items()})

@@ -184,3 +184,53 @@ def test_fusion_argument_codes(lib):
     assert call(kvshot.make_fusion_desc(num_tokens=T, hidden=D, workspace=6 * A + 16, workspace_bytes=ws)) == \
         kvshot.KVSHOT_ERR_WORKSPACE
     assert call(kvshot.make_fusion_desc(num_tokens=0, hidden=D)) == kvshot.KVSHOT_OK  # no-op
+
+
+def test_project_descriptor_layout_matches_header(tmp_path):
+    fields = [f for f, _ in kvshot.ProjectDesc._fields_]
+    src = ["#include <stdio.h>", "#include <stddef.h>", '#include "kvshot.h"', "int main(void) {",
+           'printf("%zu\\n", sizeof(kvshot_project_desc));']
+    src += [f'printf("%zu\\n", offsetof(kvshot_project_desc, {f}));' for f in fields]
+    src += ["return 0; }"]
+    c = tmp_path / "layout_project.c"
+    c.write_text("\n".join(src))
+    exe = tmp_path / "layout_project"
+    subprocess.run(["gcc", "-I", os.path.dirname(HEADER), str(c), "-o", str(exe)], check=True)
+    vals = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    assert vals[0] == ctypes.sizeof(kvshot.ProjectDesc)
+    for f, off in zip(fields, vals[1:]):
+        assert getattr(kvshot.ProjectDesc, f).offset == off, f
+
+
+def test_project_argument_codes(lib):
+    """Every case fails validation (or is the T = 0 no-op) before anything is launched."""
+    base = dict(num_tokens=4, num_layers=3, hkv=8, num_caches=2, page_size=16, max_pages_per_seq=4, num_pages=8)
+    ws = 2 * 3 * 4 * 8 * 128 * 4
+
+    def desc(**kw):
+        b = dict(base, workspace=7 * A, workspace_bytes=ws)
+        b.update(kw)
+        return kvshot.make_project_desc(**b)
+
+    def call(d, **k):
+        return kvshot.kv_project_status(d, k.get("k", A), k.get("v", 2 * A), k.get("wk", 3 * A), k.get("wv", 4 * A),
+                                        k.get("tc", 5 * A), k.get("pos", 5 * A + 256), k.get("pt", 6 * A),
+                                        k.get("ko", 8 * A), k.get("vo", 9 * A), stream=0)
+
+    assert kvshot.kv_project_workspace_size(desc()) == ws
+    assert call(None) == kvshot.KVSHOT_ERR_NULL
+    assert call(desc(num_layers=0)) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(desc(num_layers=9)) == kvshot.KVSHOT_ERR_UNSUPPORTED
+    assert call(desc(head_dim=64)) == kvshot.KVSHOT_ERR_UNSUPPORTED
+    assert call(desc(rope_base=0.0)) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(desc(num_pages=0)) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(desc(), pt=None) == kvshot.KVSHOT_ERR_SHAPE   # contiguous needs l_cap
+    assert call(desc(), k=None) == kvshot.KVSHOT_ERR_NULL
+    assert call(desc(), tc=None) == kvshot.KVSHOT_ERR_NULL
+    assert call(desc(), k=A + 8) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(desc(), pos=5 * A + 2) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(desc(workspace_bytes=ws - 1)) == kvshot.KVSHOT_ERR_WORKSPACE
+    assert call(desc(num_tokens=0)) == kvshot.KVSHOT_OK
+    d = desc()
+    d.flags = 0x2
+    assert call(d) == kvshot.KVSHOT_ERR_SHAPE
