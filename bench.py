@@ -51,9 +51,10 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--part", choices=["attn", "fusion"], default="attn",
+    ap.add_argument("--part", choices=["attn", "fusion", "project"], default="attn",
                     help="attn: the draft-attention step (default); fusion: the hybrid drafter's gated-delta "
-                         "fusion at the hybrid-tree workload's per-depth token counts")
+                         "fusion at the hybrid-tree workload's per-depth token counts; project: the KV-only "
+                         "drafter's multi-layer KV projection + RoPE fix for one step's verified tokens")
     ap.add_argument("--workload", type=int, default=5, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--mode", choices=["per_depth", "whole"], default="per_depth")
     ap.add_argument("--kernel", choices=["auto", "cc", "mma", "tc"], default="auto")
@@ -599,6 +600,132 @@ def run_fusion(args, world, rank, local):
     return result
 
 
+PROJECT_METRIC = "multi-layer KV projection tokens/s and achieved HBM GB/s (fraction of GB300 peak) at 1 GPU"
+
+
+def project_bytes(T: int, L: int, dkv: int) -> int:
+    """Algorithmic bytes of one projection call: W_K, W_V, the tokens' L-layer K/V in, their K'/V' out."""
+    return 2 * (2 * dkv * L * dkv + 2 * T * L * dkv + 2 * T * dkv)
+
+
+def run_project(args, world, rank, local):
+    """The KV-only drafter's linear projection with RoPE fix (Sec. 3.2) on the multi-layer workload's
+    shape: 4 sequences x 4 sampled target layers, 8 KV heads, paged P = 64; one call per decoding step
+    projects the step's verified tokens (here 8 per sequence, a full chain accepted) into the reused cache."""
+    from paper_2604_26412_gb300 import kvshot
+    spec = wl.config(5, seed=args.seed)
+    L, hkv, P = spec.layers, spec.hkv, spec.page_size
+    B, per_seq = spec.num_seqs, 8  # tokens verified per sequence this step (a full chain of 8 accepted)
+    T = B * per_seq
+    dkv = hkv * wl.HEAD_DIM
+    pi = wl.project_inputs(T, L, hkv, device="cuda", seed=args.seed + 7)
+    cap = 4096
+    pages_per = cap // P
+    rng = np.random.default_rng(args.seed)
+    num_pages = B * pages_per
+    page_table = torch.from_numpy(rng.permutation(num_pages).reshape(B, pages_per).astype(np.int32)).cuda()
+    token_cache = torch.arange(B, dtype=torch.int32, device="cuda").repeat_interleave(per_seq)
+    positions = (torch.arange(per_seq, dtype=torch.int32, device="cuda") + 3000).repeat(B)
+    k_pool = torch.zeros((num_pages * hkv * P, wl.HEAD_DIM), dtype=torch.bfloat16, device="cuda")
+    v_pool = torch.zeros_like(k_pool)
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    desc = kvshot.make_project_desc(num_tokens=T, num_layers=L, hkv=hkv, num_caches=B, page_size=P,
+                                    max_pages_per_seq=pages_per, num_pages=num_pages, rope_base=spec.rope_base,
+                                    rope=True, err_flag=err)
+    ws = torch.empty(kvshot.kv_project_workspace_size(desc), dtype=torch.uint8, device="cuda")
+    desc.workspace, desc.workspace_bytes = ws.data_ptr(), ws.numel()
+    stream = torch.cuda.Stream()
+    call = lambda k_in, v_in: kvshot.kv_project(desc, k_in, v_in, pi.w_k, pi.w_v, token_cache, positions, page_table,
+                                                k_pool, v_pool, stream)
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            call(pi.k_in, pi.v_in)
+    torch.cuda.synchronize()
+    graph = None
+    if not args.no_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            call(pi.k_in, pi.v_in)
+        torch.cuda.synchronize()
+    run = (lambda: graph.replay()) if graph is not None else (lambda: call(pi.k_in, pi.v_in))
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(args.steps):
+            run()
+        t1.record(stream)
+    torch.cuda.synchronize()
+    clock_info = clocks.stop()
+    barrier(world)
+    ms_total = max_over_ranks(t0.elapsed_time(t1), world)
+    assert int(err.item()) == 0, f"device error {int(err.item())}"
+    reps = 50
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(2e7))
+        for a, b in ev:
+            a.record(stream)
+            call(pi.k_in, pi.v_in)
+            b.record(stream)
+    torch.cuda.synchronize()
+    call_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    nbytes = project_bytes(T, L, dkv)
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    achieved = nbytes / (call_ms / 1e3) / 1e9
+    roofline = {"bound": "hbm", "kernel": "kvshot_kv_project (tcgen05 slab GEMM + RoPE/store kernels)",
+                "achieved": round(achieved, 1), "peak": hbm_peak, "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
+                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6.8 TB/s",
+                "traffic": None, "algorithmic_bytes_per_call": nbytes, "call_us": round(call_ms * 1e3, 2)}
+    k_h, v_h = pi.k_in.cpu().pin_memory(), pi.v_in.cpu().pin_memory()
+    k_d, v_d = torch.empty_like(pi.k_in), torch.empty_like(pi.v_in)
+    e2e_steps = max(3, min(args.steps, 100))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(e2e_steps):
+            k_d.copy_(k_h, non_blocking=True)
+            v_d.copy_(v_h, non_blocking=True)
+            call(k_d, v_d)
+            err_h = err.to("cpu", non_blocking=True)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+    result = {
+        "metric": PROJECT_METRIC, "value": round(replicas.whole_job_rate(T, args.steps, world, ms_total), 1),
+        "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_total / args.steps, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) K/V of the sampled layers, N(0,1/(L d_kv)) W_K, W_V; no trained weights)",
+        "config": {"workload": "multi-layer KV projection + RoPE fix (Sec. 3.2)", "tokens_per_call": T,
+                   "layers": L, "hkv": hkv, "layout": f"paged P={P}", "cuda_graph": graph is not None,
+                   "l2": "weights and inputs (17 MB) fit in L2; no flush (launch-bound call)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": roofline,
+        "e2e": {"value": round(replicas.whole_job_rate(T, e2e_steps, world, e2e_ms), 1), "unit": UNIT,
+                "h2d_bytes_per_step": 2 * T * L * dkv * 2, "d2h_bytes_per_step": 4},
+        "clocks": clock_info,
+        "gpu_launches": 2 * args.steps,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        from oracle import project as po
+        args_cpu = [wl.bf16_bits(x.cpu()) for x in (pi.k_in, pi.v_in, pi.w_k, pi.w_v)]
+        pos_np = positions.cpu().numpy()
+        t_start, calls = time.perf_counter(), 0
+        while time.perf_counter() - t_start < args.cpu_sample_seconds:
+            po.kv_project(*args_cpu, pos_np, spec.rope_base, True)
+            calls += 1
+        dt = time.perf_counter() - t_start
+        cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+        result["cpu_baseline"] = {"value": round(T * calls / dt, 3), "unit": UNIT, "cores": cores, "kind": "oracle",
+                                  "sample": f"{calls} projection calls of {T} tokens, fp64 oracle, {dt:.1f} s"}
+    return result
+
+
 def run_e2e(args, step, inp, stream, world):
     """Same steps through the C ABI, with the per-step inputs copied from pinned
     host buffers and the outputs copied back inside the timed region."""
@@ -664,11 +791,44 @@ def run_reference_fusion(args):
     }
 
 
+def run_reference_project(args):
+    """The projection oracle as it stands on the host cores; each step projects one decoding step's
+    verified tokens (4 sequences x 8) of the multi-layer workload."""
+    from oracle import project as po
+    spec = wl.config(5, seed=args.seed)
+    T = spec.num_seqs * 8
+    pi = wl.project_inputs(T, spec.layers, spec.hkv, device="cpu", seed=args.seed + 7)
+    a = [wl.bf16_bits(x) for x in (pi.k_in, pi.v_in, pi.w_k, pi.w_v)]
+    pos = np.tile(np.arange(8) + 3000, spec.num_seqs)
+    for _ in range(args.warmup):
+        po.kv_project(*a, pos, spec.rope_base, True)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        po.kv_project(*a, pos, spec.rope_base, True)
+    dt = time.perf_counter() - t0
+    value = T * args.steps / dt
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return {
+        "impl": "reference", "metric": PROJECT_METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; same shapes as the GPU arm)",
+        "config": {"workload": "multi-layer KV projection + RoPE fix (Sec. 3.2)", "tokens_per_call": T,
+                   "parallelism": "host cores"},
+        "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"{args.steps} projection calls of {T} tokens, fp64 oracle"},
+        "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+
+
 def run_reference(args):
     """The CPU fp64 oracle as it stands, timed on the host cores; each step is
     one drafting level (append + attention) of one sequence of the workload."""
     if args.part == "fusion":
         return run_reference_fusion(args)
+    if args.part == "project":
+        return run_reference_project(args)
     spec = wl.config(args.workload, seed=args.seed)
     samp = OracleSample(spec, args.mode, args.seed)
     for w in range(args.warmup):
@@ -712,7 +872,7 @@ def main():
         print(json.dumps(run_reference(args)), flush=True)
         return
     world, rank, local = dist_setup()
-    result = (run_fusion if args.part == "fusion" else run_ours)(args, world, rank, local)
+    result = {"fusion": run_fusion, "project": run_project}.get(args.part, run_ours)(args, world, rank, local)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:

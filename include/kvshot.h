@@ -256,7 +256,7 @@ kvshot_status kvshot_gated_delta(const kvshot_fusion_desc* desc, const void* n, 
  * All bf16 pointers 16-byte aligned, int32 pointers 4-byte aligned.  num_layers <= 8, hkv <= 64.
  * Device-side errors (a cache, position or page id out of range) skip that token's store and set
  * KVSHOT_ERR_DEVICE_BOUNDS.  T == 0 is a no-op.
- * Workspace: kvshot_kv_project_workspace_size(desc) bytes (fp32 partial products), 256-byte aligned,
+ * Workspace: kvshot_kv_project_workspace_size(desc) bytes (fp32 partial products, 8 L T d_kv bytes), 256-byte aligned,
  * no initialisation needed.
  */
 #define KVSHOT_PROJECT_ROPE 0x1u /* re-apply RoPE to the projected keys ("Proj + RoPE fix") */
