@@ -287,6 +287,23 @@ kvshot_status kvshot_kv_project(const kvshot_project_desc* desc, const void* k_i
                                 const int32_t* positions, const int32_t* page_table, void* k_out, void* v_out,
                                 kvshot_stream_t stream);
 
+/*
+ * kvshot_draft_append with QK-norm (App. D, Tab. ablations, the "QK-Norm"
+ * training regime, which the paper names without a formula; read as Qwen3's
+ * attention, which normalises q and k per head before RoPE): every
+ * 128-wide q and k head is first scaled to unit RMS and by its weights,
+ *   x <- x / sqrt(mean_j x_j^2 + eps) * w        (w = q_norm_w or k_norm_w)
+ * and then rotated exactly as kvshot_draft_append does; v is stored as is.
+ * Computed in fp32 and rounded once to bf16 (so not bit-identical to an fp64
+ * evaluation: the results are within one bf16 rounding step of it).
+ * q_norm_w, k_norm_w: [128] bf16, 4-byte aligned.  eps > 0 (Qwen3: 1e-6).
+ * Every other argument as for kvshot_draft_append.
+ */
+kvshot_status kvshot_draft_append_qknorm(const kvshot_attn_desc* desc, const void* q_in, const void* k_in,
+                                         const void* v_in, const int32_t* positions, int32_t n0, int32_t n_new,
+                                         float rope_base, const void* q_norm_w, const void* k_norm_w, float eps,
+                                         void* draft_k, void* draft_v, void* q_out, kvshot_stream_t stream);
+
 /* Static description of a status code (never NULL). */
 const char* kvshot_status_string(kvshot_status status);
 

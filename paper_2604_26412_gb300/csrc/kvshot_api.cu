@@ -326,10 +326,12 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   return e == cudaSuccess ? KVSHOT_OK : KVSHOT_ERR_CUDA;
 }
 
-extern "C" kvshot_status kvshot_draft_append(const kvshot_attn_desc* d, const void* q_in, const void* k_in,
-                                             const void* v_in, const int32_t* positions, int32_t n0,
-                                             int32_t n_new, float rope_base, void* draft_k, void* draft_v,
-                                             void* q_out, kvshot_stream_t stream) {
+namespace {
+
+kvshot_status draft_append(const kvshot_attn_desc* d, const void* q_in, const void* k_in, const void* v_in,
+                           const int32_t* positions, int32_t n0, int32_t n_new, float rope_base, const void* q_norm_w,
+                           const void* k_norm_w, float eps, void* draft_k, void* draft_v, void* q_out,
+                           kvshot_stream_t stream) {
   if (d == nullptr) return KVSHOT_ERR_NULL;
   if (d->num_caches < 1 || d->hq < 1 || d->hkv < 1 || d->n_max < 0) return KVSHOT_ERR_SHAPE;
   if (d->head_dim != kHeadDim) return KVSHOT_ERR_UNSUPPORTED;
@@ -363,6 +365,32 @@ extern "C" kvshot_status kvshot_draft_append(const kvshot_attn_desc* d, const vo
   ap.n_new = n_new;
   for (int j = 0; j < kHeadDim / 2; ++j)
     ap.inv_freq[j] = std::pow(static_cast<double>(rope_base), -2.0 * j / kHeadDim);
+  ap.q_norm_w = static_cast<const __nv_bfloat16*>(q_norm_w);
+  ap.k_norm_w = static_cast<const __nv_bfloat16*>(k_norm_w);
+  ap.eps = eps;
   const cudaError_t e = launch_append(ap, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? KVSHOT_OK : KVSHOT_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" kvshot_status kvshot_draft_append(const kvshot_attn_desc* d, const void* q_in, const void* k_in,
+                                             const void* v_in, const int32_t* positions, int32_t n0,
+                                             int32_t n_new, float rope_base, void* draft_k, void* draft_v,
+                                             void* q_out, kvshot_stream_t stream) {
+  return draft_append(d, q_in, k_in, v_in, positions, n0, n_new, rope_base, nullptr, nullptr, 0.f, draft_k, draft_v,
+                      q_out, stream);
+}
+
+extern "C" kvshot_status kvshot_draft_append_qknorm(const kvshot_attn_desc* d, const void* q_in, const void* k_in,
+                                                    const void* v_in, const int32_t* positions, int32_t n0,
+                                                    int32_t n_new, float rope_base, const void* q_norm_w,
+                                                    const void* k_norm_w, float eps, void* draft_k, void* draft_v,
+                                                    void* q_out, kvshot_stream_t stream) {
+  if (d == nullptr) return KVSHOT_ERR_NULL;
+  if (!(eps > 0.f) || !std::isfinite(eps)) return KVSHOT_ERR_SHAPE;
+  if (n_new > 0 && (q_norm_w == nullptr || k_norm_w == nullptr)) return KVSHOT_ERR_NULL;
+  if (!aligned(q_norm_w, 4) || !aligned(k_norm_w, 4)) return KVSHOT_ERR_ALIGN;
+  return draft_append(d, q_in, k_in, v_in, positions, n0, n_new, rope_base, q_norm_w, k_norm_w, eps, draft_k, draft_v,
+                      q_out, stream);
 }

@@ -81,6 +81,10 @@ struct AppendParams {
   __nv_bfloat16* q_out;
   int C, hq, hkv, n_max, n0, n_new;
   double inv_freq[kHeadDim / 2];  // rope_base^(-2j/128) in fp64
+  // QK-norm (kvshot_draft_append_qknorm): per-head RMSNorm weights over the 128 dims, or null.
+  const __nv_bfloat16* q_norm_w;
+  const __nv_bfloat16* k_norm_w;
+  float eps;
 };
 
 struct TensorMaps {
@@ -119,7 +123,7 @@ cudaError_t launch_maybe_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<Actual&&>(args)...);
 }
 cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream);
-cudaError_t launch_append(const AppendParams& a, cudaStream_t stream);
+cudaError_t launch_append(const AppendParams& a, cudaStream_t stream);  // with QK-norm when a.q_norm_w is set
 
 // CTAs per SM each kernel variant is built for (its shared-memory ring and
 // register budget are sized for this residency).

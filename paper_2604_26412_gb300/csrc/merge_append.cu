@@ -194,6 +194,66 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(const __grid_con
   }
 }
 
+// QK-norm variant (Qwen3's per-head RMSNorm of q and k before RoPE): one warp per head, lane l
+// holding dims 2l, 2l + 1 and their RoPE partners + 64.  x <- x / sqrt(mean(x^2) + eps) * w (w the
+// head-dim weights), then the rotation; fp32 throughout, one rounding to bf16.
+__global__ void __launch_bounds__(kAppendThreads) append_qknorm_kernel(const __grid_constant__ AppendParams a) {
+  if (threadIdx.x == 0) allow_dependent_launch();
+  __shared__ float s_cos[kHeadDim / 2], s_sin[kHeadDim / 2];
+  const int c = blockIdx.x / a.n_new, i = blockIdx.x - (blockIdx.x / a.n_new) * a.n_new;
+  const int pos = a.positions[static_cast<size_t>(c) * a.n_new + i];
+  for (int j = threadIdx.x; j < kHeadDim / 2; j += blockDim.x) {
+    double sn, cs;
+    sincos(static_cast<double>(pos) * a.inv_freq[j], &sn, &cs);
+    s_cos[j] = static_cast<float>(cs);
+    s_sin[j] = static_cast<float>(sn);
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j = 2 * lane;
+  for (int head = warp; head < a.hq + a.hkv; head += kAppendThreads / 32) {
+    const __nv_bfloat16* src;
+    __nv_bfloat16* dst;
+    const __nv_bfloat16* w;
+    if (head < a.hq) {
+      const size_t off = ((static_cast<size_t>(c) * a.n_new + i) * a.hq + head) * kHeadDim;
+      src = a.q_in + off;
+      dst = a.q_out + off;
+      w = a.q_norm_w;
+    } else {
+      const int kh = head - a.hq;
+      src = a.k_in + ((static_cast<size_t>(c) * a.n_new + i) * a.hkv + kh) * kHeadDim;
+      dst = a.draft_k + ((static_cast<size_t>(c) * a.hkv + kh) * a.n_max + a.n0 + i) * kHeadDim;
+      w = a.k_norm_w;
+    }
+    const uint32_t lo = *reinterpret_cast<const uint32_t*>(src + j);
+    const uint32_t hi = *reinterpret_cast<const uint32_t*>(src + 64 + j);
+    const uint32_t wl = *reinterpret_cast<const uint32_t*>(w + j);
+    const uint32_t wh = *reinterpret_cast<const uint32_t*>(w + 64 + j);
+    float x[4] = {bf16_lo(lo), bf16_hi(lo), bf16_lo(hi), bf16_hi(hi)};
+    float ss = x[0] * x[0] + x[1] * x[1] + x[2] * x[2] + x[3] * x[3];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    const float r = rsqrtf(ss * (1.f / kHeadDim) + a.eps);
+    x[0] *= r * bf16_lo(wl);
+    x[1] *= r * bf16_hi(wl);
+    x[2] *= r * bf16_lo(wh);
+    x[3] *= r * bf16_hi(wh);
+    const float c0 = s_cos[j], s0 = s_sin[j], c1 = s_cos[j + 1], s1 = s_sin[j + 1];
+    const float y0 = x[0] * c0 - x[2] * s0, y1 = x[1] * c1 - x[3] * s1;   // dims j, j + 1
+    const float z0 = x[2] * c0 + x[0] * s0, z1 = x[3] * c1 + x[1] * s1;   // dims j + 64, j + 65
+    *reinterpret_cast<uint32_t*>(dst + j) = pack_bf16x2(y0, y1);
+    *reinterpret_cast<uint32_t*>(dst + 64 + j) = pack_bf16x2(z0, z1);
+  }
+  for (int w = threadIdx.x; w < a.hkv * 16; w += blockDim.x) {  // V: plain copy into the draft slot
+    const int kh = w >> 4, ch = w & 15;
+    const uint4 v = *reinterpret_cast<const uint4*>(
+        a.v_in + ((static_cast<size_t>(c) * a.n_new + i) * a.hkv + kh) * kHeadDim + ch * 8);
+    *reinterpret_cast<uint4*>(a.draft_v + ((static_cast<size_t>(c) * a.hkv + kh) * a.n_max + a.n0 + i) * kHeadDim +
+                              ch * 8) = v;
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream) {
@@ -213,7 +273,10 @@ cudaError_t launch_merge(const AttnParams& p, cudaStream_t stream) {
 }
 
 cudaError_t launch_append(const AppendParams& a, cudaStream_t stream) {
-  append_kernel<<<a.C * a.n_new, kAppendThreads, 0, stream>>>(a);
+  if (a.q_norm_w != nullptr)
+    append_qknorm_kernel<<<a.C * a.n_new, kAppendThreads, 0, stream>>>(a);
+  else
+    append_kernel<<<a.C * a.n_new, kAppendThreads, 0, stream>>>(a);
   return cudaGetLastError();
 }
 

@@ -35,7 +35,7 @@ KVSHOT_OVERLAP_PREVIOUS = 0x10
 
 EXPORTS = ("kvshot_draft_attn", "kvshot_draft_attn_workspace_size", "kvshot_draft_append", "kvshot_status_string",
            "kvshot_version", "kvshot_draft_attn_static", "kvshot_gated_delta", "kvshot_gated_delta_workspace_size",
-           "kvshot_kv_project", "kvshot_kv_project_workspace_size")
+           "kvshot_kv_project", "kvshot_kv_project_workspace_size", "kvshot_draft_append_qknorm")
 KVSHOT_PROJECT_ROPE = 0x1
 STATIC_WORKSPACE_BYTES = 32 * 1024 * 1024  # KVSHOT_STATIC_WORKSPACE_BYTES
 
@@ -133,6 +133,9 @@ def load(build_if_missing: bool = True):
     lib.kvshot_draft_append.argtypes = [ctypes.POINTER(AttnDesc), P, P, P, P, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_float, P, P, P, P]
     lib.kvshot_draft_append.restype = ctypes.c_int
+    lib.kvshot_draft_append_qknorm.argtypes = [ctypes.POINTER(AttnDesc), P, P, P, P, ctypes.c_int32, ctypes.c_int32,
+                                               ctypes.c_float, P, P, ctypes.c_float, P, P, P, P]
+    lib.kvshot_draft_append_qknorm.restype = ctypes.c_int
     lib.kvshot_gated_delta.argtypes = [ctypes.POINTER(FusionDesc), P, P, P, P, P, P, P]
     lib.kvshot_gated_delta.restype = ctypes.c_int
     lib.kvshot_gated_delta_workspace_size.argtypes = [ctypes.POINTER(FusionDesc)]
@@ -274,3 +277,19 @@ def kv_project(desc: ProjectDesc, k_in, v_in, w_k, w_v, token_cache, positions, 
     st = kv_project_status(desc, k_in, v_in, w_k, w_v, token_cache, positions, page_table, k_out, v_out, stream)
     if st != KVSHOT_OK:
         raise KvshotError(st, "kvshot_kv_project")
+
+
+def draft_append_qknorm_status(desc: AttnDesc, q_in, k_in, v_in, positions, n0: int, n_new: int, rope_base: float,
+                               q_norm_w, k_norm_w, eps: float, draft_k, draft_v, q_out, stream=None) -> int:
+    return int(load().kvshot_draft_append_qknorm(_dref(desc), _ptr(q_in), _ptr(k_in), _ptr(v_in), _ptr(positions),
+                                                 int(n0), int(n_new), float(rope_base), _ptr(q_norm_w),
+                                                 _ptr(k_norm_w), float(eps), _ptr(draft_k), _ptr(draft_v),
+                                                 _ptr(q_out), _stream(stream)))
+
+
+def draft_append_qknorm(desc: AttnDesc, q_in, k_in, v_in, positions, n0: int, n_new: int, rope_base: float, q_norm_w,
+                        k_norm_w, eps: float, draft_k, draft_v, q_out, stream=None) -> None:
+    st = draft_append_qknorm_status(desc, q_in, k_in, v_in, positions, n0, n_new, rope_base, q_norm_w, k_norm_w, eps,
+                                    draft_k, draft_v, q_out, stream)
+    if st != KVSHOT_OK:
+        raise KvshotError(st, "kvshot_draft_append_qknorm")

@@ -141,6 +141,24 @@ def test_append_argument_codes(lib):
         kvshot.KVSHOT_ERR_UNSUPPORTED
 
 
+def test_append_qknorm_argument_codes(lib):
+    d = _desc()
+    call = lambda **k: kvshot.draft_append_qknorm_status(
+        k.get("d", d), A, A, A, A, k.get("n0", 0), k.get("n_new", 2), 1e6, k.get("wq", A), k.get("wk", A),
+        k.get("eps", 1e-6), A, A, 2 * A, stream=0)
+    assert call(d=None) == kvshot.KVSHOT_ERR_NULL
+    assert call(eps=0.0) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(eps=-1e-6) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(eps=float("nan")) == kvshot.KVSHOT_ERR_SHAPE
+    assert call(wq=None) == kvshot.KVSHOT_ERR_NULL
+    assert call(wk=None) == kvshot.KVSHOT_ERR_NULL
+    assert call(wq=A + 2) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(wk=A + 2) == kvshot.KVSHOT_ERR_ALIGN
+    assert call(n0=7) == kvshot.KVSHOT_ERR_SHAPE          # the plain append's checks apply too
+    assert call(n_new=0) == kvshot.KVSHOT_OK
+    assert call(d=_desc(head_dim=96)) == kvshot.KVSHOT_ERR_UNSUPPORTED
+
+
 def test_fusion_descriptor_layout_matches_header(tmp_path):
     fields = [f for f, _ in kvshot.FusionDesc._fields_]
     src = ["#include <stdio.h>", "#include <stddef.h>", '#include "kvshot.h"', "int main(void) {",
