@@ -114,7 +114,7 @@ extern "C" kvshot_status kvshot_gated_delta(const kvshot_fusion_desc* d, const v
   gp.err = d->err_flag;
   gp.T = T;
   gp.d_out = D;
-  gp.box_tok = std::min(T, sg::kTok);
+  gp.box_tok = std::min(T, sg::kMaxTok);
   const int nk = D / sg::kKT;
   // weight maps: 0 = W_g, 1 = W_delta; activation maps: 0 = n, 1 = o
   gp.e[0] = sg::Entry{0, 0, -1, 0, 0, 0, nk};      // W_g[:, 0:d] n

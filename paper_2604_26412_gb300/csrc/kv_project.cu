@@ -144,7 +144,7 @@ extern "C" kvshot_status kvshot_kv_project(const kvshot_project_desc* d, const v
   gp.err = d->err_flag;
   gp.T = T;
   gp.d_out = dkv;
-  gp.box_tok = std::min(T, sg::kTok);
+  gp.box_tok = std::min(T, sg::kMaxTok);
   // weight maps: 0 = W_K, 1 = W_V; activation maps: 0 = K of the L layers, 1 = V ([T, L d_kv] rows)
   for (int l = 0; l < L; ++l) {
     gp.e[l] = sg::Entry{0, 0, -1, 0, l * dkv, l * dkv, dkv / sg::kKT};

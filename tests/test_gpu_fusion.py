@@ -49,8 +49,11 @@ def _compare(h, ref, what):
     assert rel <= 3e-3, f"{what}: relative L2 error {rel:.3g}"
 
 
+# (T, d): one token; token counts that are and are not multiples of 16; 128 and 129 tokens (the
+# largest block whose n and o rows stack into one MMA, and one past it: negated-weight MMAs); 256
+# (a full block) and 257 (a second block of one token); d from 128 to 1024.
 @pytest.mark.parametrize("T,d", [(1, 128), (5, 256), (16, 384), (127, 512), (128, 256), (129, 384), (192, 1024),
-                                 (300, 512)])
+                                 (300, 512), (256, 640), (257, 128)])
 def test_fusion_matches_oracle(T, d):
     fi = wl.fusion_inputs(T, d, device="cuda", seed=T + d)
     _compare(_run(fi, T, d), _oracle(fi), f"T={T} d={d}")
