@@ -108,7 +108,7 @@ ATTN_SOURCES = ("attn_cc.cu", "attn_mma.cu", "attn_tc.cu", "kvshot_api.cu", "kvs
 
 
 # Sources of the gated-delta fusion call.
-FUSION_SOURCES = ("gated_delta.cu", "kvshot_attn_common.cuh", "kvshot_internal.h", "kvshot_tcgen05.cuh")
+FUSION_SOURCES = ("gated_delta.cu", "kvshot_slab_gemm.cuh", "kvshot_attn_common.cuh", "kvshot_internal.h", "kvshot_tcgen05.cuh")
 
 
 def kernel_source_hash(sources=ATTN_SOURCES):
