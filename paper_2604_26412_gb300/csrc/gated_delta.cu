@@ -12,9 +12,11 @@
 // one table entry each:
 //   0: W_g[:, 0:d]   n          2: W_g[:, 2d:3d] o - W_g[:, 2d:3d] n
 //   1: W_g[:, d:2d]  o          3: W_delta o - W_delta n
-// delta is never rounded to bf16: entries 2 and 3 multiply their weights by
-// n and o stacked along the token axis and subtract the two fp32 products,
-// which equals the product with the exact delta up to fp32 rounding.  Each
+// delta is never rounded to bf16: entries 2 and 3 either multiply their
+// weights by n and o stacked along the token axis and subtract the two fp32
+// products (up to 128 tokens per block), or accumulate W o and the
+// negated-weight product W n into one fp32 accumulator (larger blocks); both
+// equal the product with the exact delta up to fp32 rounding.  Each
 // product lands in a workspace slab [4][T][d].  gated_delta_finish, launched
 // behind it with programmatic stream serialization, adds the slabs and
 // applies the gate: h = n + sigmoid(slab0 + slab1 + slab2 + b_g) * slab3,
