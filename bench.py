@@ -58,6 +58,9 @@ def parse_args():
     ap.add_argument("--workload", type=int, default=5, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--mode", choices=["per_depth", "whole"], default="per_depth")
     ap.add_argument("--kernel", choices=["auto", "cc", "mma", "tc"], default="auto")
+    ap.add_argument("--kv-dtype", choices=["bf16", "fp8"], default="bf16",
+                    help="target cache element type: bf16, or fp8 e4m3 codes with power-of-two scales "
+                         "(KVSHOT_TARGET_FP8; not in the paper)")
     ap.add_argument("--num-ctas", type=int, default=0)
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -136,12 +139,13 @@ def recorded_traffic(workload, mode, kernel_hash):
     return e.get("dram_bytes_per_call")
 
 
-def algorithmic_bytes(spec: wl.Spec, n_nodes: int, n_query: int, paged: bool) -> int:
+def algorithmic_bytes(spec: wl.Spec, n_nodes: int, n_query: int, paged: bool, target_elem: int = 2) -> int:
     """Bytes one draft-attention call must move: K and V of every visible-key
     candidate (prefix + draft slots) once per KV head, q in, out and lse out,
-    the page-table entries and lengths read."""
+    the page-table entries and lengths read.  target_elem: bytes per prefix K/V
+    element (2 bf16, 1 fp8); draft K/V are bf16."""
     D = spec.head_dim
-    kv = sum(spec.hkv * (L + n_nodes) * D * 2 * 2 for L in spec.seq_lens)
+    kv = sum(spec.hkv * (L * target_elem + n_nodes * 2) * D * 2 for L in spec.seq_lens)
     qo = 2 * spec.num_caches * n_query * spec.hq * D * 2
     lse = spec.num_caches * n_query * spec.hq * 4
     pt = sum(math.ceil(L / spec.page_size) * 4 for L in spec.seq_lens) if paged else 0
@@ -292,7 +296,9 @@ def run_ours(args, world, rank, local):
     inp = wl.make_inputs(spec, dev, seed=args.seed + 1000 * rank)
     flags = {"auto": 0, "cc": kvshot.KVSHOT_FORCE_CC, "mma": kvshot.KVSHOT_FORCE_MMA,
              "tc": kvshot.KVSHOT_FORCE_TC}[args.kernel]
-    step = DraftStep(inp, mode=args.mode, flags=flags, num_ctas=args.num_ctas)
+    fp8 = args.kv_dtype == "fp8"
+    target_fp8 = (*wl.fp8_target(inp), wl.FP8_K_EXP, wl.FP8_V_EXP) if fp8 else None
+    step = DraftStep(inp, mode=args.mode, flags=flags, num_ctas=args.num_ctas, target_fp8=target_fp8)
     paged = inp.page_table is not None
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
@@ -348,20 +354,21 @@ def run_ours(args, world, rank, local):
         for r in range(reps):
             for i in range(len(levels)):
                 ev[r][i][0].record(stream)
-                kvshot.draft_attn(step.descs[i], step.q_rot[i], inp.target_k, inp.target_v, inp.page_table,
+                kvshot.draft_attn(step.descs[i], step.q_rot[i], step.target_k, step.target_v, inp.page_table,
                                   inp.seq_lens, step.draft_k, step.draft_v, step.parents[i], step.out[i], step.lse[i],
                                   stream)
                 ev[r][i][1].record(stream)
     torch.cuda.synchronize()
     call_ms = [statistics.mean(ev[r][i][0].elapsed_time(ev[r][i][1]) for r in range(reps)) for i in range(len(levels))]
-    call_bytes = [algorithmic_bytes(spec, n0s[i] + levels[i], levels[i], paged) for i in range(len(levels))]
+    call_bytes = [algorithmic_bytes(spec, n0s[i] + levels[i], levels[i], paged, 1 if fp8 else 2)
+                  for i in range(len(levels))]
     call_flops = [algorithmic_flops(spec, n0s[i] + levels[i], levels[i]) for i in range(len(levels))]
     achieved_gbs = sum(call_bytes) / (sum(call_ms) / 1e3) / 1e9
     achieved_tflops = sum(call_flops) / (sum(call_ms) / 1e3) / 1e12
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     khash = kernel_source_hash()
-    traffic = recorded_traffic(args.workload, args.mode, khash)
+    traffic = recorded_traffic(args.workload, args.mode + ("-fp8" if fp8 else ""), khash)
     rows_per_head = spec.hq // spec.hkv * max(levels)
     roofline = {
         "bound": "hbm",
@@ -395,8 +402,9 @@ def run_ours(args, world, rank, local):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "bf16",
-        "data": "synthetic (seeded N(0,1) K/V, N(0,1)/sqrt(128) q; shapes of the paper's Qwen3-8B runs)",
+        "dtype": "bf16 (target K/V fp8 e4m3)" if fp8 else "bf16",
+        "data": "synthetic (seeded N(0,1) K/V, N(0,1)/sqrt(128) q; shapes of the paper's Qwen3-8B runs)"
+                + (f"; target cache as e4m3 codes x 2^{wl.FP8_K_EXP} (K), 2^{wl.FP8_V_EXP} (V)" if fp8 else ""),
         "config": {
             "workload": spec.name,
             "mode": args.mode,
@@ -407,6 +415,7 @@ def run_ours(args, world, rank, local):
             "draft_levels": list(spec.levels),
             "tree": spec.tree,
             "layout": f"paged P={spec.page_size}" if paged else "contiguous",
+            "target_cache": "fp8 e4m3" if fp8 else "bf16",
             "gqa": f"{spec.hq}/{spec.hkv}",
             "head_dim": spec.head_dim,
             "tokens_per_step": tokens_per_step,

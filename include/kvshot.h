@@ -68,6 +68,16 @@ typedef enum kvshot_status {
  * not write seq_lens, page_table, target_k, target_v or tree_parent (kvshot_draft_append, which
  * writes q and the draft K/V, qualifies). */
 #define KVSHOT_OVERLAP_PREVIOUS 0x10u
+/* The target cache (target_k, target_v) holds fp8 E4M3 codes (OCP FP8: 1 sign bit, 4 exponent
+ * bits with bias 7, 3 mantissa bits, subnormals, codes 0x7F and 0xFF NaN, no infinities), one byte
+ * per element in the same row layout as the bf16 cache ([..][128] per token and KV head).  The
+ * key and value of a target token are decoded as
+ *   k = e4m3(code) * 2^desc->k_scale_exp,   v = e4m3(code) * 2^desc->v_scale_exp
+ * which is exact in bf16 for |exponent| <= 64; attention then proceeds as for a bf16 cache.  The
+ * draft K/V stay bf16.  Only the m16n8k16 kernel reads fp8: with this flag KVSHOT_FORCE_CC or
+ * KVSHOT_FORCE_TC returns KVSHOT_ERR_UNSUPPORTED and every stack runs on that kernel.  Not in the
+ * paper: a cache-compression variant that halves the bytes the kernel reads per target token. */
+#define KVSHOT_TARGET_FP8 0x20u
 
 /*
  * Problem descriptor shared by kvshot_draft_attn and kvshot_draft_append.
@@ -97,6 +107,8 @@ typedef struct kvshot_attn_desc {
   void* workspace;           /* device scratch, 256-byte aligned; see kvshot_draft_attn_workspace_size */
   size_t workspace_bytes;
   int32_t* err_flag;         /* optional device int32, 0 before the call; see conventions above */
+  int32_t k_scale_exp;       /* KVSHOT_TARGET_FP8: target keys are e4m3 x 2^k_scale_exp, |exp| <= 64 */
+  int32_t v_scale_exp;       /* KVSHOT_TARGET_FP8: target values are e4m3 x 2^v_scale_exp, |exp| <= 64 */
 } kvshot_attn_desc;
 
 /*

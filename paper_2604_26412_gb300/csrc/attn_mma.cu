@@ -8,6 +8,14 @@
 // softmax on the accumulator fragments, then O += P V with P re-packed from
 // the S fragments and V fragments via ldmatrix.trans.  Math as in attn_cc.cu
 // (Sec. 2.2 Eq. "kv-reattention" over M_i, Sec. 3.4 / App. B).
+//
+// A second instantiation (Cfg<..., true>) reads an fp8 e4m3 target cache
+// (KVSHOT_TARGET_FP8): the TMA brings each target tile's codes into the upper
+// half of its K and V tiles, the consumer warps expand every tile to f16 in
+// shared memory, and all MMAs run in f16 with the cache's power-of-two scales
+// folded into the score scale and into P.
+#include <cuda_fp16.h>
+
 #include "kvshot_attn_common.cuh"
 
 namespace kvshot {
@@ -15,11 +23,53 @@ namespace {
 
 using namespace dev;
 
+// With an fp8 target cache (KVSHOT_TARGET_FP8) the kernel multiplies in f16: e4m3 -> f16 is exact
+// (3 mantissa bits, exponents inside f16's range) and one conversion instruction per pair; q, the
+// draft tiles and P are rounded to f16 (more mantissa than bf16; only values below 2^-14 lose
+// bits).  The cache's power-of-two scales are folded into the score scale (keys) and into P
+// (values), so one set of MMA fragments serves both kinds of tile.
+// Four e4m3 codes (a 32-bit word, lowest byte first) -> four f16 values (two f16x2 words).
+__device__ __forceinline__ uint2 e4m3x4_to_f16x4(uint32_t codes) {
+  uint2 r;
+  asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %2;\n\t"
+      "cvt.rn.f16x2.e4m3x2 %0, lo;\n\tcvt.rn.f16x2.e4m3x2 %1, hi;\n\t}"
+      : "=r"(r.x), "=r"(r.y)
+      : "r"(codes));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t w) { return pack_f16x2(bf16_lo(w), bf16_hi(w)); }
+
+__device__ __forceinline__ uint4 bf16x8_to_f16x8(uint4 v) {
+  return make_uint4(bf16x2_to_f16x2(v.x), bf16x2_to_f16x2(v.y), bf16x2_to_f16x2(v.z), bf16x2_to_f16x2(v.w));
+}
+
+// 8 consecutive codes (dims 8ch .. 8ch+7 of one row) -> one 16-byte f16 chunk.
+__device__ __forceinline__ uint4 expand8(const uint2 codes) {
+  const uint2 lo = e4m3x4_to_f16x4(codes.x), hi = e4m3x4_to_f16x4(codes.y);
+  return make_uint4(lo.x, lo.y, hi.x, hi.y);
+}
+
+// D += A * B, m16n8k16, f16 inputs, fp32 accumulate.
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
 constexpr int kBarConsumers = 1;
 constexpr int kCombStride = kHeadDim + 4;  // padded fp32 row in the combine buffer
 
-template <int MT, int KS, int STAGES, int MINB>
+template <int MT, int KS, int STAGES, int MINB, bool F8 = false>
 struct Cfg {
+  static constexpr bool kF8 = F8;                     // fp8 target tiles (KVSHOT_TARGET_FP8)
   static constexpr int kMT = MT;                      // m16 tiles per unit
   static constexpr int kKS = KS;                      // key slices per tile
   static constexpr int kStages = STAGES;
@@ -185,7 +235,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
   const int mt = warp % CF::kMT, ks = warp / CF::kMT;
   const int g = lane >> 2, q4 = lane & 3;
   const int HR = p.hkv * p.row_blocks;
-  uint32_t qa[8][4];
+  uint32_t qa[8][4];  // bf16 pairs, or f16 pairs in the fp8 variant
   float o[16][4];
   float m_run[2], l_run[2];
   int stage = 0;
@@ -211,6 +261,12 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
           qa[kk][2 + i] = ok ? src[kk * 8 + 4 + q4] : 0u;  // dims 16kk + 8 + 2q4, +1
         }
       }
+      if constexpr (CF::kF8) {
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+#pragma unroll
+          for (int r = 0; r < 4; ++r) qa[kk][r] = bf16x2_to_f16x2(qa[kk][r]);
+      }
 #pragma unroll
       for (int nd = 0; nd < 16; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
       m_run[0] = m_run[1] = -INFINITY;
@@ -231,6 +287,43 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
     uint8_t* kptr = pipe.ring + static_cast<size_t>(stage) * kStageBytes;
     const uint32_t kbase = smem_addr(kptr);
     const uint32_t vbase = kbase + kKVTileBytes;
+    const bool f16t = CF::kF8 && !ti.draft;  // this tile's K/V are fp8 codes (scaled by 2^exp)
+    if constexpr (CF::kF8) {
+      // fp8 variant: every tile becomes f16 in place.  Target tiles: the e4m3 rows (128 bytes per
+      // key) sit in the upper half of the K and V tiles; a row's upper f16 half lands exactly on that
+      // row's codes, which the 16 lanes converting the row have all loaded before the warp stores.
+      // Draft tiles: each 16-byte chunk of 8 bf16 is rewritten as 8 f16.  With one m-tile per unit
+      // each warp reads only the K and V rows of its own key slice, so it converts just those and
+      // no barrier is needed (except before the tail rows are zeroed).
+      constexpr bool kOwnRows = CF::kMT == 1;
+      const int row0 = kOwnRows ? ks * CF::kKW : 0;            // first key row this warp converts
+      const int nrows = kOwnRows ? CF::kKW : kTileKeys;        // key rows per K (and per V) tile
+      const int w0 = kOwnRows ? 0 : warp, wstep = kOwnRows ? 1 : CF::kWarps;
+      if (__all_sync(0xffffffffu, live)) {
+        if (f16t) {
+          // Two rows per warp instruction: lane = (row parity, 16-byte chunk ch) takes the row's codes
+          // 8ch .. 8ch+7, so the 16 lanes of a row read it whole (8 bytes each) and write its 16
+          // chunks, which the 128-byte swizzle spreads over all banks.
+          for (int g2 = w0; g2 < nrows; g2 += wstep) {
+            const int r = g2 * 2 + (lane >> 4);  // K rows, then V rows
+            const int kv = r / nrows, key = row0 + r % nrows, ch = lane & 15;
+            uint8_t* tile = kptr + kv * kKVTileBytes;
+            const uint2 codes = *reinterpret_cast<const uint2*>(tile + kHalfBytes + key * 128 + ch * 8);
+            __syncwarp();
+            *reinterpret_cast<uint4*>(tile + tile_off(key, ch)) = expand8(codes);
+          }
+        } else {
+          for (int i = w0 * 32 + lane; i < 2 * nrows * 16; i += wstep * 32) {
+            const int r = i / 16, ch = i % 16;
+            uint4* chunk =
+                reinterpret_cast<uint4*>(kptr + (r / nrows) * kKVTileBytes + tile_off(row0 + r % nrows, ch));
+            *chunk = bf16x8_to_f16x8(*chunk);
+          }
+        }
+        fence_proxy_async_smem();  // the next TMA write into this stage comes after these stores
+      }
+      if (!kOwnRows || ti.nkeys < kTileKeys) named_barrier_sync(kBarConsumers, CF::kWarps * 32);
+    }
     if (ti.nkeys < kTileKeys) {
       // V rows past the valid keys may be stale or NaN; the P.V product would
       // spread a NaN through 0 * NaN, so zero them (all consumer threads).
@@ -258,11 +351,17 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
         for (int kp = 0; kp < 4; ++kp) {
           uint32_t b0, b1, b2, b3;
           ldmatrix_x4(kbase + tile_off(key, kp * 4 + lmat), b0, b1, b2, b3);
-          mma_bf16_16816(s[j], qa[2 * kp], b0, b1);
-          mma_bf16_16816(s[j], qa[2 * kp + 1], b2, b3);
+          if constexpr (CF::kF8) {
+            mma_f16_16816(s[j], qa[2 * kp], b0, b1);
+            mma_f16_16816(s[j], qa[2 * kp + 1], b2, b3);
+          } else {
+            mma_bf16_16816(s[j], qa[2 * kp], b0, b1);
+            mma_bf16_16816(s[j], qa[2 * kp + 1], b2, b3);
+          }
         }
       }
       // Scale into the log2 domain, mask, row max over this warp's keys.
+      const float qs = f16t ? p.qscale * p.k_scale : p.qscale;
       float mx[2] = {-INFINITY, -INFINITY};
 #pragma unroll
       for (int j = 0; j < CF::kNT; ++j) {
@@ -272,7 +371,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
           const int rl = rl0 + (e >> 1) * 8;
           bool valid = key < ti.nkeys;
           if (ti.draft) valid = valid && draft_visible(p, sm.anc, rb * p.rows_per_unit + rl, ti.key0 + key);
-          s[j][e] = valid ? s[j][e] * p.qscale : -INFINITY;
+          s[j][e] = valid ? s[j][e] * qs : -INFINITY;
           mx[e >> 1] = fmaxf(mx[e >> 1], s[j][e]);
         }
       }
@@ -311,17 +410,30 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
 #pragma unroll
       for (int kk = 0; kk < CF::kNT / 2; ++kk) {
         uint32_t pa[4];
-        pa[0] = pack_bf16x2(s[2 * kk][0], s[2 * kk][1]);
-        pa[1] = pack_bf16x2(s[2 * kk][2], s[2 * kk][3]);
-        pa[2] = pack_bf16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-        pa[3] = pack_bf16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+        if constexpr (CF::kF8) {  // P times the value scale, in f16 (the running sum keeps the unscaled P)
+          const float vs = f16t ? p.v_scale : 1.f;
+          pa[0] = pack_f16x2(s[2 * kk][0] * vs, s[2 * kk][1] * vs);
+          pa[1] = pack_f16x2(s[2 * kk][2] * vs, s[2 * kk][3] * vs);
+          pa[2] = pack_f16x2(s[2 * kk + 1][0] * vs, s[2 * kk + 1][1] * vs);
+          pa[3] = pack_f16x2(s[2 * kk + 1][2] * vs, s[2 * kk + 1][3] * vs);
+        } else {
+          pa[0] = pack_bf16x2(s[2 * kk][0], s[2 * kk][1]);
+          pa[1] = pack_bf16x2(s[2 * kk][2], s[2 * kk][3]);
+          pa[2] = pack_bf16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+          pa[3] = pack_bf16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+        }
         const int key = kw0 + kk * 16 + ((lmat & 1) << 3) + lrow;
 #pragma unroll
         for (int ndp = 0; ndp < 8; ++ndp) {
           uint32_t b0, b1, b2, b3;
           ldmatrix_x4_trans(vbase + tile_off(key, 2 * ndp + (lmat >> 1)), b0, b1, b2, b3);
-          mma_bf16_16816(o[2 * ndp], pa, b0, b1);
-          mma_bf16_16816(o[2 * ndp + 1], pa, b2, b3);
+          if constexpr (CF::kF8) {
+            mma_f16_16816(o[2 * ndp], pa, b0, b1);
+            mma_f16_16816(o[2 * ndp + 1], pa, b2, b3);
+          } else {
+            mma_bf16_16816(o[2 * ndp], pa, b0, b1);
+            mma_bf16_16816(o[2 * ndp + 1], pa, b2, b3);
+          }
         }
       }
     }
@@ -377,10 +489,10 @@ __global__ void __launch_bounds__(CF::kThreads, CF::kMinBlocks)
   if (threadIdx.x == 0) drain_after_abort(p, pipe, sm.misc[2]);
 }
 
-using Cfg1 = Cfg<1, 4, 3, 2>;
-using Cfg2 = Cfg<2, 4, 4, 1>;
-using Cfg3 = Cfg<3, 2, 4, 1>;
-using Cfg4 = Cfg<4, 2, 4, 1>;
+template <bool F8> using Cfg1 = Cfg<1, 4, 3, 2, F8>;
+template <bool F8> using Cfg2 = Cfg<2, 4, 4, 1, F8>;
+template <bool F8> using Cfg3 = Cfg<3, 2, 4, 1, F8>;
+template <bool F8> using Cfg4 = Cfg<4, 2, 4, 1, F8>;
 
 template <class CF>
 cudaError_t launch_cfg(const AttnParams& p, const TensorMaps& maps, bool pdl, cudaStream_t stream) {
@@ -402,26 +514,36 @@ cudaError_t occupancy_cfg(int C, int* ctas) {
 
 }  // namespace
 
-int attn_mma_ctas_per_sm(int m_tiles) { return m_tiles == 1 ? Cfg1::kMinBlocks : 1; }
+int attn_mma_ctas_per_sm(int m_tiles) { return m_tiles == 1 ? Cfg1<false>::kMinBlocks : 1; }
 
-cudaError_t attn_mma_occupancy(int m_tiles, int C, int* ctas_per_sm) {
+template <bool F8>
+cudaError_t occupancy_f8(int m_tiles, int C, int* ctas_per_sm) {
   switch (m_tiles) {
-    case 1: return occupancy_cfg<Cfg1>(C, ctas_per_sm);
-    case 2: return occupancy_cfg<Cfg2>(C, ctas_per_sm);
-    case 3: return occupancy_cfg<Cfg3>(C, ctas_per_sm);
-    case 4: return occupancy_cfg<Cfg4>(C, ctas_per_sm);
+    case 1: return occupancy_cfg<Cfg1<F8>>(C, ctas_per_sm);
+    case 2: return occupancy_cfg<Cfg2<F8>>(C, ctas_per_sm);
+    case 3: return occupancy_cfg<Cfg3<F8>>(C, ctas_per_sm);
+    case 4: return occupancy_cfg<Cfg4<F8>>(C, ctas_per_sm);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t attn_mma_occupancy(int m_tiles, int C, bool fp8, int* ctas_per_sm) {
+  return fp8 ? occupancy_f8<true>(m_tiles, C, ctas_per_sm) : occupancy_f8<false>(m_tiles, C, ctas_per_sm);
+}
+
+template <bool F8>
+cudaError_t launch_f8(const AttnParams& p, const TensorMaps& maps, int m_tiles, bool pdl, cudaStream_t stream) {
+  switch (m_tiles) {
+    case 1: return launch_cfg<Cfg1<F8>>(p, maps, pdl, stream);
+    case 2: return launch_cfg<Cfg2<F8>>(p, maps, pdl, stream);
+    case 3: return launch_cfg<Cfg3<F8>>(p, maps, pdl, stream);
+    case 4: return launch_cfg<Cfg4<F8>>(p, maps, pdl, stream);
     default: return cudaErrorInvalidValue;
   }
 }
 
 cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, bool pdl, cudaStream_t stream) {
-  switch (m_tiles) {
-    case 1: return launch_cfg<Cfg1>(p, maps, pdl, stream);
-    case 2: return launch_cfg<Cfg2>(p, maps, pdl, stream);
-    case 3: return launch_cfg<Cfg3>(p, maps, pdl, stream);
-    case 4: return launch_cfg<Cfg4>(p, maps, pdl, stream);
-    default: return cudaErrorInvalidValue;
-  }
+  return p.fp8 ? launch_f8<true>(p, maps, m_tiles, pdl, stream) : launch_f8<false>(p, maps, m_tiles, pdl, stream);
 }
 
 }  // namespace kvshot

@@ -15,7 +15,7 @@ namespace kvshot {
 
 // Defined in the kernel translation units.
 cudaError_t attn_cc_occupancy(int C, int* ctas_per_sm);
-cudaError_t attn_mma_occupancy(int m_tiles, int C, int* ctas_per_sm);
+cudaError_t attn_mma_occupancy(int m_tiles, int C, bool fp8, int* ctas_per_sm);
 cudaError_t attn_tc_occupancy(int C, int* ctas_per_sm);
 
 namespace {
@@ -52,6 +52,22 @@ bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
+
+// fp8 E4M3 target cache: one byte per element, whole 128-byte rows per box, no swizzle (the
+// m16n8k16 kernel expands each tile to the bf16 layout in shared memory).
+bool encode_rows_fp8(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(kHeadDim)};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kHeadDim), box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+constexpr int kMaxScaleExp = 64;
 
 enum class Kernel { kCudaCore, kMma, kTensorMemory };
 
@@ -124,8 +140,15 @@ kvshot_status check_common(const kvshot_attn_desc* d) {
   if (d->n_nodes < 0 || d->n_query < 0 || d->n_query > d->n_nodes || d->n_nodes > d->n_max) return KVSHOT_ERR_SHAPE;
   if (d->max_seq_len < 0) return KVSHOT_ERR_SHAPE;
   if (!std::isfinite(d->scale)) return KVSHOT_ERR_SHAPE;
-  const uint32_t known = KVSHOT_TREE | KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC | KVSHOT_OVERLAP_PREVIOUS;
+  const uint32_t known =
+      KVSHOT_TREE | KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC | KVSHOT_OVERLAP_PREVIOUS | KVSHOT_TARGET_FP8;
   if ((d->flags & ~known) != 0) return KVSHOT_ERR_SHAPE;
+  if (d->flags & KVSHOT_TARGET_FP8) {
+    if (d->k_scale_exp < -kMaxScaleExp || d->k_scale_exp > kMaxScaleExp || d->v_scale_exp < -kMaxScaleExp ||
+        d->v_scale_exp > kMaxScaleExp)
+      return KVSHOT_ERR_SHAPE;
+    if (d->flags & (KVSHOT_FORCE_CC | KVSHOT_FORCE_TC)) return KVSHOT_ERR_UNSUPPORTED;  // m16n8k16 kernel only
+  }
   const uint32_t force = d->flags & (KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC);
   if (force & (force - 1)) return KVSHOT_ERR_SHAPE;  // at most one kernel may be forced
   const int G = d->hq / d->hkv;
@@ -168,7 +191,8 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   //    shared memory into tensor memory, is faster (1.5x at 48 rows, 3-4x for
   //    whole-tree stacks of 128-256 rows).
   const bool tc_ok = G <= 128 && 128 % G == 0;
-  const Kernel automatic = (rows > 16 && tc_ok) ? Kernel::kTensorMemory : Kernel::kMma;
+  const bool fp8 = d->flags & KVSHOT_TARGET_FP8;  // only the m16n8k16 kernel expands fp8 tiles
+  const Kernel automatic = (rows > 16 && tc_ok && !fp8) ? Kernel::kTensorMemory : Kernel::kMma;
   pl->kernel = force_cc ? Kernel::kCudaCore : force_tc ? Kernel::kTensorMemory
                                            : force_mma ? Kernel::kMma : automatic;
   pl->mma = pl->kernel == Kernel::kMma;
@@ -199,7 +223,7 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   int grid = d->num_ctas;
   if (grid == 0) {
     int per_sm = 0;
-    const cudaError_t e = pl->kernel == Kernel::kMma ? attn_mma_occupancy(pl->m_tiles, d->num_caches, &per_sm)
+    const cudaError_t e = pl->kernel == Kernel::kMma ? attn_mma_occupancy(pl->m_tiles, d->num_caches, fp8, &per_sm)
                           : pl->kernel == Kernel::kTensorMemory ? attn_tc_occupancy(d->num_caches, &per_sm)
                                                                  : attn_cc_occupancy(d->num_caches, &per_sm);
     const int sms = sm_count();
@@ -271,8 +295,12 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
                                : static_cast<uint64_t>(d->num_caches) * d->hkv * d->l_cap;
   const uint32_t tbox = paged ? static_cast<uint32_t>(std::min(d->page_size, kTileKeys)) : kTileKeys;
   const uint64_t drows = static_cast<uint64_t>(d->num_caches) * d->hkv * d->n_max;
-  if (!encode_rows(&maps.tk, target_k, trows, tbox) || !encode_rows(&maps.tv, target_v, trows, tbox) ||
-      !encode_rows(&maps.dk, draft_k, drows, kDraftBoxRows) || !encode_rows(&maps.dv, draft_v, drows, kDraftBoxRows))
+  const bool fp8 = (d->flags & KVSHOT_TARGET_FP8) != 0;
+  const bool tmaps = fp8 ? encode_rows_fp8(&maps.tk, target_k, trows, tbox) &&
+                               encode_rows_fp8(&maps.tv, target_v, trows, tbox)
+                         : encode_rows(&maps.tk, target_k, trows, tbox) && encode_rows(&maps.tv, target_v, trows, tbox);
+  if (!tmaps || !encode_rows(&maps.dk, draft_k, drows, kDraftBoxRows) ||
+      !encode_rows(&maps.dv, draft_v, drows, kDraftBoxRows))
     return KVSHOT_ERR_CUDA;
   if (pl.kernel == Kernel::kTensorMemory) {
     if (!encode_q(&maps.q, q, d->num_caches, d->n_query, d->hq, q_box(d->hq / d->hkv, pl.nq_box, pl.spread)))
@@ -315,6 +343,9 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   const double scale = d->scale != 0.f ? static_cast<double>(d->scale) : 1.0 / std::sqrt(static_cast<double>(kHeadDim));
   p.qscale = static_cast<float>(scale * 1.4426950408889634);
   p.num_ctas = pl.num_ctas;
+  p.fp8 = fp8 ? 1 : 0;
+  p.k_scale = fp8 ? std::ldexp(1.f, d->k_scale_exp) : 1.f;
+  p.v_scale = fp8 ? std::ldexp(1.f, d->v_scale_exp) : 1.f;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const bool pdl = (d->flags & KVSHOT_OVERLAP_PREVIOUS) != 0;

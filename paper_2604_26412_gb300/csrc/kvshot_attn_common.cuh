@@ -498,23 +498,27 @@ __device__ __forceinline__ void run_producer(const AttnParams& p, const TensorMa
                       full_bar, policy);
         }
       } else if (p.paged) {
+        // bf16: boxes of 64 dims per half; fp8 (p.fp8): one box of whole 128-byte rows, into the
+        // upper half of the tile (the lanes of half 1 skip), expanded there by the consumers.
         const int br = p.box_rows;
         const int nbox = (nkeys + br - 1) / br;
-        if (lane == 0) mbar_arrive_expect_tx(full_bar, nbox * br * 128 * 4);
-        if (i < nbox) {
+        if (lane == 0) mbar_arrive_expect_tx(full_bar, nbox * br * 128 * (p.fp8 ? 2 : 4));
+        if (i < nbox && !(p.fp8 && hf)) {
           int pid = pids[0];
 #pragma unroll
           for (int k = 1; k < kTileKeys / 8; ++k)
             if (i == k) pid = pids[k];
           const int krow = key0 + i * br;
           const int y = (pid * p.hkv + h) * p.page_size + (krow % p.page_size);
-          tma_load_2d(dst + i * br * 128, kv ? &maps.tv : &maps.tk, hf * 64, y, full_bar, policy);
+          const uint32_t d0 = p.fp8 ? kdst + kv * kKVTileBytes + kHalfBytes : dst;
+          tma_load_2d(d0 + i * br * 128, kv ? &maps.tv : &maps.tk, p.fp8 ? 0 : hf * 64, y, full_bar, policy);
         }
       } else {
-        if (lane == 0) mbar_arrive_expect_tx(full_bar, kTileKeys * 128 * 4);
-        if (i == 0) {
+        if (lane == 0) mbar_arrive_expect_tx(full_bar, kTileKeys * 128 * (p.fp8 ? 2 : 4));
+        if (i == 0 && !(p.fp8 && hf)) {
           const int y = (cu.c * p.hkv + h) * p.l_cap + key0;
-          tma_load_2d(dst, kv ? &maps.tv : &maps.tk, hf * 64, y, full_bar, policy);
+          const uint32_t d0 = p.fp8 ? kdst + kv * kKVTileBytes + kHalfBytes : dst;
+          tma_load_2d(d0, kv ? &maps.tv : &maps.tk, p.fp8 ? 0 : hf * 64, y, full_bar, policy);
         }
       }
     }

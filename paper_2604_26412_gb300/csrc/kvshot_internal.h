@@ -69,6 +69,8 @@ struct AttnParams {
   int draft_tiles;          // ceil(N / TK)
   float qscale;             // softmax scale * log2(e): scores are kept in the log2 domain
   int num_ctas;             // persistent grid size
+  int fp8;                  // target K/V are e4m3 codes (KVSHOT_TARGET_FP8; m16n8k16 kernel only)
+  float k_scale, v_scale;   // fp8: 2^k_scale_exp, 2^v_scale_exp
 };
 
 struct AppendParams {

@@ -32,6 +32,7 @@ KVSHOT_FORCE_CC = 0x2
 KVSHOT_FORCE_MMA = 0x4
 KVSHOT_FORCE_TC = 0x8
 KVSHOT_OVERLAP_PREVIOUS = 0x10
+KVSHOT_TARGET_FP8 = 0x20
 
 EXPORTS = ("kvshot_draft_attn", "kvshot_draft_attn_workspace_size", "kvshot_draft_append", "kvshot_status_string",
            "kvshot_version", "kvshot_draft_attn_static", "kvshot_gated_delta", "kvshot_gated_delta_workspace_size",
@@ -69,6 +70,8 @@ class AttnDesc(ctypes.Structure):
         ("workspace", ctypes.c_void_p),
         ("workspace_bytes", ctypes.c_size_t),
         ("err_flag", ctypes.c_void_p),
+        ("k_scale_exp", ctypes.c_int32),
+        ("v_scale_exp", ctypes.c_int32),
     ]
 
 
@@ -184,11 +187,11 @@ def _stream(stream) -> Optional[int]:
 
 def make_desc(*, num_caches, num_seqs, hq, hkv, n_nodes, n_query, n_max, max_seq_len, head_dim=128, page_size=0,
               max_pages_per_seq=0, num_pages=0, l_cap=0, scale=0.0, tree=False, flags=0, num_ctas=0,
-              workspace=None, workspace_bytes=0, err_flag=None) -> AttnDesc:
+              workspace=None, workspace_bytes=0, err_flag=None, k_scale_exp=0, v_scale_exp=0) -> AttnDesc:
     f = int(flags) | (KVSHOT_TREE if tree else 0)
     return AttnDesc(num_caches, num_seqs, hq, hkv, head_dim, page_size, max_pages_per_seq, num_pages, l_cap,
                     max_seq_len, n_nodes, n_query, n_max, float(scale), f, num_ctas, _ptr(workspace),
-                    int(workspace_bytes), _ptr(err_flag))
+                    int(workspace_bytes), _ptr(err_flag), int(k_scale_exp), int(v_scale_exp))
 
 
 def workspace_size(desc: AttnDesc) -> int:

@@ -21,11 +21,19 @@ from . import workloads as wl
 
 class DraftStep:
     def __init__(self, inp: wl.Inputs, mode: str = "per_depth", flags: int = 0, num_ctas: int = 0,
-                 scale: float = 0.0, err_flag: bool = True):
+                 scale: float = 0.0, err_flag: bool = True, target_fp8=None):
+        """target_fp8: optional (codes_k, codes_v, k_scale_exp, v_scale_exp), an e4m3 copy of the target
+        cache (workloads.fp8_target) to attend instead of inp.target_k / inp.target_v."""
         if mode not in ("per_depth", "whole"):
             raise ValueError(mode)
         self.inp, self.mode = inp, mode
         s = inp.spec
+        k_exp = v_exp = 0
+        if target_fp8 is not None:
+            self.target_k, self.target_v, k_exp, v_exp = target_fp8
+            flags |= kvshot.KVSHOT_TARGET_FP8
+        else:
+            self.target_k, self.target_v = inp.target_k, inp.target_v
         dev = inp.target_k.device
         self.device = dev
         C, N = s.num_caches, s.n_nodes
@@ -58,7 +66,8 @@ class DraftStep:
                 max_pages_per_seq=inp.page_table.shape[1] if paged else 0,
                 num_pages=inp.num_pages if paged else 0, l_cap=inp.l_cap, scale=scale, tree=s.tree,
                 # the attention call follows this step's own append kernel, which writes only q and the draft K/V
-                flags=flags | kvshot.KVSHOT_OVERLAP_PREVIOUS, num_ctas=num_ctas, err_flag=self.err))
+                flags=flags | kvshot.KVSHOT_OVERLAP_PREVIOUS, num_ctas=num_ctas, err_flag=self.err,
+                k_scale_exp=k_exp, v_scale_exp=v_exp))
         ws = max(kvshot.workspace_size(d) for d in self.descs)
         if ws == 0:
             raise kvshot.KvshotError(kvshot.KVSHOT_ERR_SHAPE, "kvshot_draft_attn_workspace_size")
@@ -79,7 +88,7 @@ class DraftStep:
             d = self.descs[i]
             kvshot.draft_append(d, self.q_in[i], self.k_in[i], self.v_in[i], self.pos[i], n0, n_step,
                                 inp.spec.rope_base, self.draft_k, self.draft_v, self.q_rot[i], stream)
-            kvshot.draft_attn(d, self.q_rot[i], inp.target_k, inp.target_v, inp.page_table, inp.seq_lens,
+            kvshot.draft_attn(d, self.q_rot[i], self.target_k, self.target_v, inp.page_table, inp.seq_lens,
                               self.draft_k, self.draft_v, self.parents[i], self.out[i], self.lse[i], stream)
             n0 += n_step
 

@@ -215,6 +215,21 @@ def _fill_tails(spec, tk, tv, page_table, lens, value):
             tv[c, :, int(L):, :] = value
 
 
+# Scale exponents of the fp8 target-cache variant: keys and values are cached as e4m3 codes of
+# x / 2^exp, so that N(0, 1) entries use the middle of e4m3's range (|x| 2^3 stays far below 448).
+FP8_K_EXP = -3
+FP8_V_EXP = -2
+
+
+def fp8_target(inp: Inputs, k_exp: int = FP8_K_EXP, v_exp: int = FP8_V_EXP):
+    """e4m3 codes (uint8 tensors shaped like target_k) of target_k / 2^k_exp and target_v / 2^v_exp,
+    rounded to nearest by torch's float8_e4m3fn conversion (NaN entries stay NaN codes).  This is
+    how a target model would fill an fp8 cache; the library only reads the codes."""
+    def enc(x, e):
+        return (x.float() * 2.0 ** (-e)).to(torch.float8_e4m3fn).view(torch.uint8).contiguous()
+    return enc(inp.target_k, k_exp), enc(inp.target_v, v_exp)
+
+
 def draft_buffers(spec: Spec, n_max: int, device="cpu", fill: float = float("nan")):
     """Empty draft K/V buffers [C, hkv, n_max, D] pre-filled with `fill` (NaN by default,
     so reading an unwritten slot is caught)."""

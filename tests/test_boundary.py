@@ -96,7 +96,11 @@ def _attn(d, **ptrs):
     (dict(num_pages=0), kvshot.KVSHOT_ERR_SHAPE),
     (dict(max_seq_len=-1), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=0x80), kvshot.KVSHOT_ERR_SHAPE),
-    (dict(flags=0x20), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(flags=0x40), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(flags=kvshot.KVSHOT_TARGET_FP8, k_scale_exp=65), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(flags=kvshot.KVSHOT_TARGET_FP8, v_scale_exp=-65), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(flags=kvshot.KVSHOT_TARGET_FP8 | kvshot.KVSHOT_FORCE_TC), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    (dict(flags=kvshot.KVSHOT_TARGET_FP8 | kvshot.KVSHOT_FORCE_CC), kvshot.KVSHOT_ERR_UNSUPPORTED),
     (dict(flags=kvshot.KVSHOT_FORCE_CC | kvshot.KVSHOT_FORCE_MMA), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=kvshot.KVSHOT_FORCE_MMA | kvshot.KVSHOT_FORCE_TC), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=kvshot.KVSHOT_FORCE_TC, hq=24, hkv=8), kvshot.KVSHOT_ERR_UNSUPPORTED),
