@@ -735,40 +735,69 @@ def run_project(args, world, rank, local):
     return result
 
 
+def _arena(tensors, device):
+    """One device buffer holding every tensor (256-byte aligned slots) and views of it shaped like
+    them; returns (buffer, views, total bytes)."""
+    offs, off = [], 0
+    for t in tensors:
+        offs.append(off)
+        off += (t.numel() * t.element_size() + 255) // 256 * 256
+    buf = torch.empty(max(off, 256), dtype=torch.uint8, device=device)
+    views = [buf[o:o + t.numel() * t.element_size()].view(t.dtype).view(t.shape) for o, t in zip(offs, tensors)]
+    return buf, views, off
+
+
 def run_e2e(args, step, inp, stream, world):
-    """Same steps through the C ABI, with the per-step inputs copied from pinned
-    host buffers and the outputs copied back inside the timed region."""
-    host_in = []
-    dev_in = []
+    """Same steps through the C ABI, with the per-step inputs copied from pinned host memory and
+    the outputs copied back inside the timed region.  A serving loop would keep a step's inputs in
+    one host arena: the step's device inputs (q/k/v/positions of every level, parents, lengths,
+    page table) are views of one device buffer filled by one copy per step, and its outputs
+    (out and lse of every level) views of one buffer read back by one copy."""
+    import dataclasses
+    ins = [t for lst in (step.q_in, step.k_in, step.v_in, step.pos) for t in lst] + list(step.parents) + \
+        [inp.seq_lens] + ([inp.page_table] if inp.page_table is not None else [])
+    dbuf_in, views_in, h2d = _arena(ins, ins[0].device)
+    for v, t in zip(views_in, ins):
+        v.copy_(t)
+    k = 0
     for lst in (step.q_in, step.k_in, step.v_in, step.pos):
-        for t in lst:
-            host_in.append(t.cpu().pin_memory())
-            dev_in.append(t)
-    for t in step.parents + [inp.seq_lens] + ([inp.page_table] if inp.page_table is not None else []):
-        host_in.append(t.cpu().pin_memory())
-        dev_in.append(t)
-    host_out = [t.cpu().pin_memory() for t in step.out + step.lse]
-    dev_out = step.out + step.lse
-    h2d = sum(t.numel() * t.element_size() for t in host_in)
-    d2h = sum(t.numel() * t.element_size() for t in host_out)
+        for i in range(len(lst)):
+            lst[i] = views_in[k]
+            k += 1
+    for i in range(len(step.parents)):
+        step.parents[i] = views_in[k]
+        k += 1
+    inp_e2e = dataclasses.replace(inp, seq_lens=views_in[k],
+                                  page_table=views_in[k + 1] if inp.page_table is not None else None)
+    inp_saved, step.inp = step.inp, inp_e2e
+    outs = list(step.out) + list(step.lse)
+    dbuf_out, views_out, d2h = _arena(outs, outs[0].device)
+    nl = len(step.out)
+    step.out = views_out[:nl]
+    step.lse = views_out[nl:]
+    host_in = dbuf_in.cpu().pin_memory()
+    host_out = torch.empty(dbuf_out.numel(), dtype=torch.uint8).pin_memory()
     steps = max(3, min(args.steps, 100))
+    with torch.cuda.stream(stream):  # one untimed pass through the new buffers
+        dbuf_in.copy_(host_in, non_blocking=True)
+        step.run()
     torch.cuda.synchronize()
     barrier(world)
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         a.record(stream)
         for _ in range(steps):
-            for h, d in zip(host_in, dev_in):
-                d.copy_(h, non_blocking=True)
+            dbuf_in.copy_(host_in, non_blocking=True)
             step.run()
-            for d, h in zip(dev_out, host_out):
-                h.copy_(d, non_blocking=True)
+            host_out.copy_(dbuf_out, non_blocking=True)
         b.record(stream)
     torch.cuda.synchronize()
+    step.inp = inp_saved
     ms = max_over_ranks(a.elapsed_time(b), world)
     value = replicas.whole_job_rate(step.tokens, steps, world, ms)
     return {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-            "steps": steps, "api": "kvshot_draft_append + kvshot_draft_attn via ctypes, no CUDA graph"}
+            "steps": steps, "api": "kvshot_draft_append + kvshot_draft_attn via ctypes, no CUDA graph; "
+                                   "inputs and outputs in one pinned host arena each (one copy each way per step)"}
 
 
 # --------------------------------------------------------- reference arm
