@@ -89,7 +89,9 @@ def test_gate_extremes():
 
 def test_workspace_reuse_and_garbage():
     # The workspace needs no initialisation: fill it with NaN bit patterns and reuse it across shapes.
-    ws = torch.full((16 * 300 * 1024,), 0xFF, dtype=torch.uint8, device="cuda")
-    for T, d in ((300, 512), (7, 1024), (130, 256)):
+    shapes = ((300, 512), (7, 1024), (130, 256))
+    need = max(kvshot.gated_delta_workspace_size(kvshot.make_fusion_desc(num_tokens=T, hidden=d)) for T, d in shapes)
+    ws = torch.full((need,), 0xFF, dtype=torch.uint8, device="cuda")
+    for T, d in shapes:
         fi = wl.fusion_inputs(T, d, device="cuda", seed=T)
         _compare(_run(fi, T, d, ws=ws), _oracle(fi), f"reused workspace T={T} d={d}")
