@@ -211,6 +211,27 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
 // 0..15, so every SM sub-partition's softmax warps get rows; two threads share
 // a lane (row), each with 32 of the 64 columns, and agree on the row max by
 // one shuffle.
+// O_wg *= alpha (per row) in TMEM, after P.V of this warpgroup's previous tile (t - 2) completed.
+template <bool kSpread>
+__device__ __forceinline__ void rescale_o_tmem(const Smem& sm, const Pipe& pipe, const AttnParams& p, uint32_t my_o,
+                                               int t, float alpha) {
+  constexpr int kOChunks = kSpread ? 2 : 4;  // 32-column O chunks per thread
+  if (!mbar_wait(smem_addr(&sm.pvdone[(t - 2) % kNP]), ((t - 2) / kNP) & 1, p.err)) *pipe.abort = 1;
+  tc_fence_after();
+#pragma unroll
+  for (int c = 0; c < kOChunks; ++c) {
+    uint32_t o[32];
+    if constexpr (kSpread) tmem_ld16x2_32(my_o + 32 * c, o);
+    else tmem_ld32(my_o + 32 * c, o);
+    tmem_wait_ld();
+#pragma unroll
+    for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha);
+    if constexpr (kSpread) tmem_st16x2_32(my_o + 32 * c, o);
+    else tmem_st32(my_o + 32 * c, o);
+  }
+  tmem_wait_st();
+}
+
 template <bool kSpread>
 __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                             Cursor cu) {
@@ -275,6 +296,8 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       live = __all_sync(0xffffffffu, live);
       tc_fence_after();
       float pr[kCols];
+      bool any_rescale = false;  // dense rows: some row of this warp moves its reference max, O_wg is rescaled
+      float alpha = 1.f;         // dense rows: this row's factor
       if (!(live && warp_live)) mbar_arrive(smem_addr(&sm.sfree[sbuf]));  // S is not read
       if (live && warp_live) {
         uint32_t sv[kCols];
@@ -311,26 +334,21 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         }
         float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
         if constexpr (kSpread) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-        // Lazy rescale: move this row's reference max only when it grows by > 2^8.
+        // Lazy rescale: move this row's reference max only when it grows by > 2^8.  Dense rows rescale
+        // O_wg after P is stored (below), so that P's 64 registers are free by then (it removed the
+        // dense variant's spills); spread rows, with half the columns, rescale here, which measured
+        // faster for them.
         const bool grow = valid && (m_run == -INFINITY ? mx != -INFINITY : mx > m_run + kRescaleThreshold);
         const bool rescale_o = grow && m_run != -INFINITY;
-        if (__any_sync(0xffffffffu, rescale_o)) {
-          // O_wg must hold P.V of this warpgroup's previous tile (t - 2) before it is scaled.
-          if (!mbar_wait(smem_addr(&sm.pvdone[(t - 2) % kNP]), ((t - 2) / kNP) & 1, p.err)) *pipe.abort = 1;
-          tc_fence_after();
-          const float alpha = rescale_o ? ex2(m_run - mx) : 1.f;
-#pragma unroll
-          for (int c = 0; c < kOChunks; ++c) {
-            uint32_t o[32];
-            if constexpr (kSpread) tmem_ld16x2_32(my_o + 32 * c, o);
-            else tmem_ld32(my_o + 32 * c, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha);
-            if constexpr (kSpread) tmem_st16x2_32(my_o + 32 * c, o);
-            else tmem_st32(my_o + 32 * c, o);
+        if constexpr (kSpread) {
+          if (__any_sync(0xffffffffu, rescale_o)) {
+            const float a = rescale_o ? ex2(m_run - mx) : 1.f;
+            rescale_o_tmem<kSpread>(sm, pipe, p, my_o, t, a);
+            l_run *= a;
           }
-          tmem_wait_st();
+        } else {
+          any_rescale = __any_sync(0xffffffffu, rescale_o);
+          alpha = rescale_o ? ex2(m_run - mx) : 1.f;
           l_run *= alpha;
         }
         if (grow) m_run = mx;
@@ -357,6 +375,9 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
           w.w = pack_bf16x2(pr[8 * c + 6], pr[8 * c + 7]);
           *reinterpret_cast<uint4*>(prow + ((chunk ^ (tl & 7)) << 4)) = w;
         }
+      }
+      if constexpr (!kSpread) {
+        if (live && warp_live && any_rescale) rescale_o_tmem<kSpread>(sm, pipe, p, my_o, t, alpha);
       }
       if (live && ti.nkeys < kTileKeys) {
         // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.
