@@ -1,0 +1,44 @@
+"""The benchmark's byte and rate arithmetic (the roofline's numerator), checked by hand; no GPU."""
+import math
+
+import bench
+from paper_2604_26412_gb300 import replicas
+from paper_2604_26412_gb300 import workloads as wl
+
+
+def _spec(lens, levels, tree, paged, P=16, hq=32, hkv=8):
+    return wl.Spec("t", len(lens), 1, list(lens), list(levels), tree, paged, page_size=P, hq=hq, hkv=hkv, seed=0)
+
+
+def test_attention_bytes_by_hand():
+    # one cache, 100 prefix tokens, 3 draft nodes of which 2 query, paged P = 16, chain
+    s = _spec([100], [1, 2], False, True)
+    D, hkv, hq = 128, 8, 32
+    kv = hkv * (100 + 3) * D * 2 * 2                 # K and V of every visible-key candidate, bf16
+    qo = 2 * 1 * 2 * hq * D * 2                      # q in, out out
+    lse = 1 * 2 * hq * 4
+    pt = math.ceil(100 / 16) * 4
+    meta = 1 * 4                                     # seq_lens (no tree parents for a chain)
+    assert bench.algorithmic_bytes(s, 3, 2, True) == kv + qo + lse + pt + meta
+
+
+def test_fp8_target_bytes_halve_only_the_prefix():
+    s = _spec([1000, 24], [4, 4], True, False)
+    b16 = bench.algorithmic_bytes(s, 8, 4, False)
+    b8 = bench.algorithmic_bytes(s, 8, 4, False, target_elem=1)
+    # only the prefix K/V shrink: 1024 tokens x 8 heads x 128 dims x (K, V) x 1 byte
+    assert b16 - b8 == (1000 + 24) * 8 * 128 * 2
+    tree_meta = 2 * 8 * 4
+    assert b16 - bench.algorithmic_bytes(_spec([1000, 24], [4, 4], False, False), 8, 4, False) == tree_meta
+
+
+def test_flops_and_fusion_bytes():
+    s = _spec([64], [2], False, True, hq=4, hkv=1)
+    assert bench.algorithmic_flops(s, 2, 2) == 4 * 4 * 2 * (64 + 2) * 128
+    d, T = 256, 3
+    assert bench.fusion_bytes(T, d) == 2 * (4 * d * d + d + 3 * T * d)
+
+
+def test_whole_job_rate_counts_every_rank_against_the_slowest():
+    assert replicas.whole_job_rate(100, steps=10, world=1, max_ms=2.0) == 500_000.0
+    assert replicas.whole_job_rate(100, steps=10, world=4, max_ms=2.0) == 2_000_000.0
