@@ -58,6 +58,8 @@ def parse_args():
     ap.add_argument("--workload", type=int, default=5, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--mode", choices=["per_depth", "whole"], default="per_depth")
     ap.add_argument("--kernel", choices=["auto", "cc", "mma", "tc"], default="auto")
+    ap.add_argument("--qk-norm", action="store_true",
+                    help="the append normalises q and k per head before RoPE (kvshot_draft_append_qknorm)")
     ap.add_argument("--kv-dtype", choices=["bf16", "fp8"], default="bf16",
                     help="target cache element type: bf16, or fp8 e4m3 codes with power-of-two scales "
                          "(KVSHOT_TARGET_FP8; not in the paper)")
@@ -298,7 +300,13 @@ def run_ours(args, world, rank, local):
              "tc": kvshot.KVSHOT_FORCE_TC}[args.kernel]
     fp8 = args.kv_dtype == "fp8"
     target_fp8 = (*wl.fp8_target(inp), wl.FP8_K_EXP, wl.FP8_V_EXP) if fp8 else None
-    step = DraftStep(inp, mode=args.mode, flags=flags, num_ctas=args.num_ctas, target_fp8=target_fp8)
+    qk_norm = None
+    if args.qk_norm:  # synthetic per-dimension weights around 1, Qwen3's eps
+        g = torch.Generator().manual_seed(args.seed + 17)
+        qk_norm = tuple((0.5 + torch.rand(spec.head_dim, generator=g)).to(torch.bfloat16).to(dev) for _ in range(2)) \
+            + (1e-6,)
+    step = DraftStep(inp, mode=args.mode, flags=flags, num_ctas=args.num_ctas, target_fp8=target_fp8,
+                     qk_norm=qk_norm)
     paged = inp.page_table is not None
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
@@ -416,6 +424,7 @@ def run_ours(args, world, rank, local):
             "tree": spec.tree,
             "layout": f"paged P={spec.page_size}" if paged else "contiguous",
             "target_cache": "fp8 e4m3" if fp8 else "bf16",
+            "append": "QK-norm + RoPE" if args.qk_norm else "RoPE",
             "gqa": f"{spec.hq}/{spec.hkv}",
             "head_dim": spec.head_dim,
             "tokens_per_step": tokens_per_step,

@@ -21,12 +21,15 @@ from . import workloads as wl
 
 class DraftStep:
     def __init__(self, inp: wl.Inputs, mode: str = "per_depth", flags: int = 0, num_ctas: int = 0,
-                 scale: float = 0.0, err_flag: bool = True, target_fp8=None):
+                 scale: float = 0.0, err_flag: bool = True, target_fp8=None, qk_norm=None):
         """target_fp8: optional (codes_k, codes_v, k_scale_exp, v_scale_exp), an e4m3 copy of the target
-        cache (workloads.fp8_target) to attend instead of inp.target_k / inp.target_v."""
+        cache (workloads.fp8_target) to attend instead of inp.target_k / inp.target_v.
+        qk_norm: optional (q_norm_w, k_norm_w, eps): the append normalises q and k per head first
+        (kvshot_draft_append_qknorm)."""
         if mode not in ("per_depth", "whole"):
             raise ValueError(mode)
         self.inp, self.mode = inp, mode
+        self.qk_norm = qk_norm
         s = inp.spec
         k_exp = v_exp = 0
         if target_fp8 is not None:
@@ -86,8 +89,14 @@ class DraftStep:
         n0 = 0
         for i, n_step in enumerate(self.levels):
             d = self.descs[i]
-            kvshot.draft_append(d, self.q_in[i], self.k_in[i], self.v_in[i], self.pos[i], n0, n_step,
-                                inp.spec.rope_base, self.draft_k, self.draft_v, self.q_rot[i], stream)
+            if self.qk_norm is not None:
+                wq, wk, eps = self.qk_norm
+                kvshot.draft_append_qknorm(d, self.q_in[i], self.k_in[i], self.v_in[i], self.pos[i], n0, n_step,
+                                           inp.spec.rope_base, wq, wk, eps, self.draft_k, self.draft_v,
+                                           self.q_rot[i], stream)
+            else:
+                kvshot.draft_append(d, self.q_in[i], self.k_in[i], self.v_in[i], self.pos[i], n0, n_step,
+                                    inp.spec.rope_base, self.draft_k, self.draft_v, self.q_rot[i], stream)
             kvshot.draft_attn(d, self.q_rot[i], self.target_k, self.target_v, inp.page_table, inp.seq_lens,
                               self.draft_k, self.draft_v, self.parents[i], self.out[i], self.lse[i], stream)
             n0 += n_step

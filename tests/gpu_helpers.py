@@ -56,6 +56,20 @@ def oracle_attn(hc: HostCache, q, draft_k, draft_v, n_nodes, n_query, caches=Non
                        dk, dv, par)
 
 
+def round_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round fp64 to the nearest bf16 (ties to even), as uint16 bit patterns, in exact integer arithmetic."""
+    m, e = np.frexp(x)                      # x = m 2^e, 0.5 <= |m| < 1
+    q = np.ldexp(m, 8)                       # 8 significant bits: |q| in [128, 256)
+    r = np.rint(q)                           # numpy rounds half to even
+    y = np.ldexp(r, e - 8).astype(np.float32)  # exact: at most 8 significant bits
+    return (y.view(np.uint32) >> 16).astype(np.uint16)
+
+
+def widen_bits(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns to fp64, exactly."""
+    return (np.asarray(bits).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
 def compare(out_gpu: torch.Tensor, lse_gpu: torch.Tensor, out_ref: np.ndarray, lse_ref: np.ndarray, what=""):
     """Assert the tolerances; returns (max_abs, rel_l2, lse_err)."""
     o = out_gpu.float().cpu().numpy().astype(np.float64)

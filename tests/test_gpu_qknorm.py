@@ -16,22 +16,10 @@ import torch
 from oracle import qknorm as qo
 from paper_2604_26412_gb300 import kvshot
 from paper_2604_26412_gb300 import workloads as wl
+from tests.gpu_helpers import round_bf16_bits as _round_bf16, widen_bits as _widen
 
 pytestmark = pytest.mark.gpu
 D = 128
-
-
-def _round_bf16(x: np.ndarray) -> np.ndarray:
-    """Round fp64 to the nearest bf16 (ties to even), as bit patterns, in exact integer arithmetic."""
-    m, e = np.frexp(x)                      # x = m 2^e, 0.5 <= |m| < 1
-    q = np.ldexp(m, 8)                       # 8 significant bits: |q| in [128, 256)
-    r = np.rint(q)                           # numpy rounds half to even
-    y = np.ldexp(r, e - 8).astype(np.float32)  # exact: at most 8 significant bits
-    return (y.view(np.uint32) >> 16).astype(np.uint16)
-
-
-def _widen(bits: np.ndarray) -> np.ndarray:
-    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
 def _case(C, hq, hkv, n_new, n0, n_max, max_pos, seed, in_place=False, eps=1e-6):

@@ -100,3 +100,43 @@ def test_append_is_bit_exact_at_long_positions():
     kvshot.draft_append(d, q_in, k_in, v_in, pos, n0, n_new, spec.rope_base, dk, dv, q_in)
     torch.cuda.synchronize()
     assert np.array_equal(wl.bf16_bits(q_in), q_ref)
+
+
+@pytest.mark.parametrize("cfg,caches", [(2, None), (5, [1, 10])])
+def test_step_with_qknorm_matches_oracle(cfg, caches):
+    """The step with the QK-norm append (kvshot_draft_append_qknorm) against the oracle's QK-norm append and
+    attention.  The append rounds once from fp32, so q and k are within one bf16 step of the fp64 values; the
+    attention is held to the usual tolerances on the oracle's own rounded q and k."""
+    from oracle import qknorm as qo
+    spec = wl.config(cfg, seed=0)
+    inp = wl.make_inputs(spec, "cuda")
+    g = torch.Generator().manual_seed(23)
+    wq = (0.5 + torch.rand(spec.head_dim, generator=g)).to(torch.bfloat16)
+    wk = (0.5 + torch.rand(spec.head_dim, generator=g)).to(torch.bfloat16)
+    eps = 1e-6
+    step = DraftStep(inp, mode="per_depth", qk_norm=(wq.cuda(), wk.cuda(), eps))
+    step.run()
+    torch.cuda.synchronize()
+    assert step.error_code() == 0
+    hc = gh.HostCache(inp)
+    sel = list(range(spec.num_caches)) if caches is None else caches
+    C, D = spec.num_caches, spec.head_dim
+    dk = np.full((C, spec.hkv, inp.n_max, D), 0x7FC0, np.uint16)
+    dv = dk.copy()
+    n0 = 0
+    for i, n_step in enumerate(spec.levels):
+        qr, kr, vr = qo.append_qknorm(wl.bf16_bits(inp.q_in[i]), wl.bf16_bits(inp.k_in[i]), wl.bf16_bits(inp.v_in[i]),
+                                      inp.positions[i].cpu().numpy(), n0, spec.rope_base, wl.bf16_bits(wq),
+                                      wl.bf16_bits(wk), eps, inp.n_max)
+        dk[:, :, n0:n0 + n_step] = gh.round_bf16_bits(kr)
+        dv[:, :, n0:n0 + n_step] = gh.round_bf16_bits(vr)
+        n0 += n_step
+        gq = gh.widen_bits(wl.bf16_bits(step.q_rot[i]))
+        assert np.all(np.abs(gq - qr) <= 2.0 ** -8 * np.abs(qr) + 1e-5), f"level {i}: q off by more than a bf16 step"
+        out, lse = gh.oracle_attn(hc, wl.bits_to_bf16(gh.round_bf16_bits(qr)), wl.bits_to_bf16(dk),
+                                  wl.bits_to_bf16(dv), n0, n_step, caches=caches)
+        gh.compare(step.out[i][sel], step.lse[i][sel], out, lse, f"cfg{cfg} qk-norm level {i}")
+    gk = gh.widen_bits(wl.bf16_bits(step.draft_k)[:, :, :n0])
+    rk = gh.widen_bits(dk[:, :, :n0])
+    assert np.all(np.abs(gk - rk) <= 2.0 ** -7 * np.abs(rk) + 1e-5)
+    assert np.array_equal(wl.bf16_bits(step.draft_v)[:, :, :n0], dv[:, :, :n0])
