@@ -10,10 +10,18 @@
 // (Sec. 2.2 Eq. "kv-reattention" over M_i, Sec. 3.4 / App. B).
 //
 // A second instantiation (Cfg<..., true>) reads an fp8 e4m3 target cache
-// (KVSHOT_TARGET_FP8): the TMA brings each target tile's codes into the upper
-// half of its K and V tiles, the consumer warps expand every tile to f16 in
-// shared memory, and all MMAs run in f16 with the cache's power-of-two scales
-// folded into the score scale and into P.
+// (KVSHOT_TARGET_FP8): the TMA brings each target tile's codes (128-byte rows,
+// 128B-swizzled) into the upper half of its K and V tiles, and the consumer
+// warps decode them straight into MMA fragments in registers; all MMAs run in
+// f16 with the cache's power-of-two scales folded into the score scale and
+// into P.  Fragment layouts of that variant: a lane's 16-byte load of one key
+// row feeds four k-steps of S = Q K^T, so the head dimensions of q are taken
+// in the same permuted order (k-step 4h + s, pair position 2 q4 -> dims
+// 16 (2 q4 + h) + 4 s + {0, 1}, position 8 + 2 q4 -> + {2, 3}); for O += P V a
+// lane pairs the same 16 dims of two key rows with byte permutes, so the
+// output columns are permuted too (n8 tile nd, column n -> dim 16 n + nd) and
+// the write-out undoes it.  Draft tiles (bf16) are read into the same layouts
+// and converted to f16 in registers.
 #include <cuda_fp16.h>
 
 #include "kvshot_attn_common.cuh"
@@ -45,14 +53,22 @@ __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
 
 __device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t w) { return pack_f16x2(bf16_lo(w), bf16_hi(w)); }
 
-__device__ __forceinline__ uint4 bf16x8_to_f16x8(uint4 v) {
-  return make_uint4(bf16x2_to_f16x2(v.x), bf16x2_to_f16x2(v.y), bf16x2_to_f16x2(v.z), bf16x2_to_f16x2(v.w));
+// 16 bytes from shared memory (ordered after the pipeline's barrier waits like the ldmatrix loads).
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+  return v;
 }
 
-// 8 consecutive codes (dims 8ch .. 8ch+7 of one row) -> one 16-byte f16 chunk.
-__device__ __forceinline__ uint4 expand8(const uint2 codes) {
-  const uint2 lo = e4m3x4_to_f16x4(codes.x), hi = e4m3x4_to_f16x4(codes.y);
-  return make_uint4(lo.x, lo.y, hi.x, hi.y);
+// Word t (0..3) of a 16-byte vector; t is a compile-time constant after unrolling.
+__device__ __forceinline__ uint32_t word(const uint4& v, int t) {
+  return t == 0 ? v.x : t == 1 ? v.y : t == 2 ? v.z : v.w;
+}
+
+// Byte offset, inside a K or V tile, of 16-byte chunk c (0..7: dims 16c .. 16c+15) of fp8 key row r:
+// the codes occupy the tile's upper half as 128-byte rows under the TMA's 128-byte swizzle.
+__device__ __forceinline__ uint32_t code_off(int r, int c) {
+  return static_cast<uint32_t>(kHalfBytes + r * 128 + ((c ^ (r & 7)) << 4));
 }
 
 // D += A * B, m16n8k16, f16 inputs, fp32 accumulate.
@@ -205,7 +221,38 @@ __device__ __forceinline__ void finalize(const AttnParams& p, const Smem& sm, in
           if (rl >= p.rows_per_unit || rr >= p.rows_total) continue;
           const float inv = Lsum[i] > 0.f ? 1.f / Lsum[i] : 0.f;
           const float lse2 = Lsum[i] > 0.f ? M[i] + __log2f(Lsum[i]) : -INFINITY;
-          if (whole) {
+          if constexpr (CF::kF8) {
+            // Permuted columns: o[nd][2i] is dim 32 q4 + nd, o[nd][2i + 1] dim 32 q4 + 16 + nd, so the
+            // lane owns dims 32 q4 .. 32 q4 + 31 of the row and writes them as 16-byte vectors.
+            if (whole) {
+              const int nl = rr / p.G, gh = rr - nl * p.G;
+              const size_t row = (static_cast<size_t>(c) * p.Nq + nl) * p.hq + h * p.G + gh;
+              uint4* dst = reinterpret_cast<uint4*>(p.out + row * kHeadDim + 32 * q4);
+#pragma unroll
+              for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+                for (int v = 0; v < 2; ++v) {
+                  const int e = 2 * i + hh, n0 = 8 * v;
+                  dst[2 * hh + v] = make_uint4(pack_bf16x2(o[n0][e] * inv, o[n0 + 1][e] * inv),
+                                               pack_bf16x2(o[n0 + 2][e] * inv, o[n0 + 3][e] * inv),
+                                               pack_bf16x2(o[n0 + 4][e] * inv, o[n0 + 5][e] * inv),
+                                               pack_bf16x2(o[n0 + 6][e] * inv, o[n0 + 7][e] * inv));
+                }
+              if (q4 == 0) p.lse[row] = lse2 * 0.69314718055994531f;
+            } else {
+              const size_t row = static_cast<size_t>(slot) * p.rows_per_unit + rl;
+              float4* dst = reinterpret_cast<float4*>(p.ws_o + row * kHeadDim + 32 * q4);
+#pragma unroll
+              for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+                for (int v = 0; v < 4; ++v) {
+                  const int e = 2 * i + hh, n0 = 4 * v;
+                  dst[4 * hh + v] = make_float4(o[n0][e] * inv, o[n0 + 1][e] * inv, o[n0 + 2][e] * inv,
+                                                o[n0 + 3][e] * inv);
+                }
+              if (q4 == 0) p.ws_lse[row] = lse2;
+            }
+          } else if (whole) {
             const int nl = rr / p.G, gh = rr - nl * p.G;
             const size_t row = (static_cast<size_t>(c) * p.Nq + nl) * p.hq + h * p.G + gh;
             __nv_bfloat16* dst = p.out + row * kHeadDim + 2 * q4;
@@ -241,12 +288,14 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
   int stage = 0;
   uint32_t phase = 0;
   int piece_lt0 = 0, anc_seq = -1, consumed = 0;
+  int h = 0, rb = 0;  // KV head and row block of the current piece
 
   for (; cu.t < cu.t_end; cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
-    const int h = cu.hr / p.row_blocks, rb = cu.hr - (cu.hr / p.row_blocks) * p.row_blocks;
     const int rl0 = mt * 16 + g;                       // rows of this thread within the unit
     if (ti.first) {
+      h = cu.hr / p.row_blocks;
+      rb = cu.hr - h * p.row_blocks;
       piece_lt0 = cu.lt;
 #pragma unroll
       for (int i = 0; i < 2; ++i) {
@@ -257,15 +306,15 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
             p.q + ((static_cast<size_t>(cu.c) * p.Nq + nl) * p.hq + h * p.G + gh) * kHeadDim);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          qa[kk][i] = ok ? src[kk * 8 + q4] : 0u;          // dims 16kk + 2q4, +1
-          qa[kk][2 + i] = ok ? src[kk * 8 + 4 + q4] : 0u;  // dims 16kk + 8 + 2q4, +1
+          if constexpr (CF::kF8) {  // f16, k-step 4h + s on dims 16 (2 q4 + h) + 4 s + {0..3}
+            const int w = 8 * (2 * q4 + (kk >> 2)) + 2 * (kk & 3);
+            qa[kk][i] = ok ? bf16x2_to_f16x2(src[w]) : 0u;
+            qa[kk][2 + i] = ok ? bf16x2_to_f16x2(src[w + 1]) : 0u;
+          } else {
+            qa[kk][i] = ok ? src[kk * 8 + q4] : 0u;          // dims 16kk + 2q4, +1
+            qa[kk][2 + i] = ok ? src[kk * 8 + 4 + q4] : 0u;  // dims 16kk + 8 + 2q4, +1
+          }
         }
-      }
-      if constexpr (CF::kF8) {
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-#pragma unroll
-          for (int r = 0; r < 4; ++r) qa[kk][r] = bf16x2_to_f16x2(qa[kk][r]);
       }
 #pragma unroll
       for (int nd = 0; nd < 16; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
@@ -288,45 +337,10 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
     const uint32_t kbase = smem_addr(kptr);
     const uint32_t vbase = kbase + kKVTileBytes;
     const bool f16t = CF::kF8 && !ti.draft;  // this tile's K/V are fp8 codes (scaled by 2^exp)
-    if constexpr (CF::kF8) {
-      // fp8 variant: every tile becomes f16 in place.  Target tiles: the e4m3 rows (128 bytes per
-      // key) sit in the upper half of the K and V tiles; a row's upper f16 half lands exactly on that
-      // row's codes, which the 16 lanes converting the row have all loaded before the warp stores.
-      // Draft tiles: each 16-byte chunk of 8 bf16 is rewritten as 8 f16.  With one m-tile per unit
-      // each warp reads only the K and V rows of its own key slice, so it converts just those and
-      // no barrier is needed (except before the tail rows are zeroed).
-      constexpr bool kOwnRows = CF::kMT == 1;
-      const int row0 = kOwnRows ? ks * CF::kKW : 0;            // first key row this warp converts
-      const int nrows = kOwnRows ? CF::kKW : kTileKeys;        // key rows per K (and per V) tile
-      const int w0 = kOwnRows ? 0 : warp, wstep = kOwnRows ? 1 : CF::kWarps;
-      if (__all_sync(0xffffffffu, live)) {
-        if (f16t) {
-          // Two rows per warp instruction: lane = (row parity, 16-byte chunk ch) takes the row's codes
-          // 8ch .. 8ch+7, so the 16 lanes of a row read it whole (8 bytes each) and write its 16
-          // chunks, which the 128-byte swizzle spreads over all banks.
-          for (int g2 = w0; g2 < nrows; g2 += wstep) {
-            const int r = g2 * 2 + (lane >> 4);  // K rows, then V rows
-            const int kv = r / nrows, key = row0 + r % nrows, ch = lane & 15;
-            uint8_t* tile = kptr + kv * kKVTileBytes;
-            const uint2 codes = *reinterpret_cast<const uint2*>(tile + kHalfBytes + key * 128 + ch * 8);
-            __syncwarp();
-            *reinterpret_cast<uint4*>(tile + tile_off(key, ch)) = expand8(codes);
-          }
-        } else {
-          for (int i = w0 * 32 + lane; i < 2 * nrows * 16; i += wstep * 32) {
-            const int r = i / 16, ch = i % 16;
-            uint4* chunk =
-                reinterpret_cast<uint4*>(kptr + (r / nrows) * kKVTileBytes + tile_off(row0 + r % nrows, ch));
-            *chunk = bf16x8_to_f16x8(*chunk);
-          }
-        }
-        fence_proxy_async_smem();  // the next TMA write into this stage comes after these stores
-      }
-      if (!kOwnRows || ti.nkeys < kTileKeys) named_barrier_sync(kBarConsumers, CF::kWarps * 32);
-    }
-    if (ti.nkeys < kTileKeys) {
+    if (!CF::kF8 && ti.nkeys < kTileKeys) {
       // V rows past the valid keys may be stale or NaN; the P.V product would
-      // spread a NaN through 0 * NaN, so zero them (all consumer threads).
+      // spread a NaN through 0 * NaN, so zero them (all consumer threads).  The
+      // fp8 variant drops those rows in registers instead.
       if (live) {
         uint8_t* vptr = kptr + kKVTileBytes;
         const int nz = (kTileKeys - ti.nkeys) * 16;  // 16-byte chunks to clear
@@ -344,17 +358,47 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
 #pragma unroll
       for (int j = 0; j < CF::kNT; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
       const int lrow = lane & 7, lmat = lane >> 3;
+      if constexpr (CF::kF8) {
+        // Lane (g, q4) reads dims 16 (2 q4 + kh) .. + 15 of key row kw0 + 8j + g: four k-steps' B
+        // fragments.  Under the swizzle the two rows of each 8-lane phase take chunks of opposite
+        // parity, so the loads are free of bank conflicts.  Two accumulators per n8 tile (one per kh)
+        // halve the MMA dependency chain.
+        float s2[CF::kNT][4];
 #pragma unroll
-      for (int j = 0; j < CF::kNT; ++j) {
-        const int key = kw0 + j * 8 + lrow;
+        for (int j = 0; j < CF::kNT; ++j) {
+          s2[j][0] = s2[j][1] = s2[j][2] = s2[j][3] = 0.f;
+          const int key = kw0 + j * 8 + g;
 #pragma unroll
-        for (int kp = 0; kp < 4; ++kp) {
-          uint32_t b0, b1, b2, b3;
-          ldmatrix_x4(kbase + tile_off(key, kp * 4 + lmat), b0, b1, b2, b3);
-          if constexpr (CF::kF8) {
-            mma_f16_16816(s[j], qa[2 * kp], b0, b1);
-            mma_f16_16816(s[j], qa[2 * kp + 1], b2, b3);
-          } else {
+          for (int kh = 0; kh < 2; ++kh) {
+            const int c = 2 * q4 + kh;
+            uint32_t b[8];
+            if (f16t) {
+              const uint4 w = lds128(kbase + code_off(key, c));
+              const uint2 f0 = e4m3x4_to_f16x4(w.x), f1 = e4m3x4_to_f16x4(w.y);
+              const uint2 f2 = e4m3x4_to_f16x4(w.z), f3 = e4m3x4_to_f16x4(w.w);
+              b[0] = f0.x; b[1] = f0.y; b[2] = f1.x; b[3] = f1.y;
+              b[4] = f2.x; b[5] = f2.y; b[6] = f3.x; b[7] = f3.y;
+            } else {
+              const uint4 lo = lds128(kbase + tile_off(key, 2 * c)), hi = lds128(kbase + tile_off(key, 2 * c + 1));
+              b[0] = bf16x2_to_f16x2(lo.x); b[1] = bf16x2_to_f16x2(lo.y);
+              b[2] = bf16x2_to_f16x2(lo.z); b[3] = bf16x2_to_f16x2(lo.w);
+              b[4] = bf16x2_to_f16x2(hi.x); b[5] = bf16x2_to_f16x2(hi.y);
+              b[6] = bf16x2_to_f16x2(hi.z); b[7] = bf16x2_to_f16x2(hi.w);
+            }
+#pragma unroll
+            for (int st = 0; st < 4; ++st) mma_f16_16816(kh ? s2[j] : s[j], qa[4 * kh + st], b[2 * st], b[2 * st + 1]);
+          }
+#pragma unroll
+          for (int e = 0; e < 4; ++e) s[j][e] += s2[j][e];
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < CF::kNT; ++j) {
+          const int key = kw0 + j * 8 + lrow;
+#pragma unroll
+          for (int kp = 0; kp < 4; ++kp) {
+            uint32_t b0, b1, b2, b3;
+            ldmatrix_x4(kbase + tile_off(key, kp * 4 + lmat), b0, b1, b2, b3);
             mma_bf16_16816(s[j], qa[2 * kp], b0, b1);
             mma_bf16_16816(s[j], qa[2 * kp + 1], b2, b3);
           }
@@ -363,16 +407,26 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
       // Scale into the log2 domain, mask, row max over this warp's keys.
       const float qs = f16t ? p.qscale * p.k_scale : p.qscale;
       float mx[2] = {-INFINITY, -INFINITY};
+      if (!ti.draft && ti.nkeys == kTileKeys) {  // a full prefix tile: every key is visible
 #pragma unroll
-      for (int j = 0; j < CF::kNT; ++j) {
+        for (int j = 0; j < CF::kNT; ++j)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int key = kw0 + j * 8 + 2 * q4 + (e & 1);
-          const int rl = rl0 + (e >> 1) * 8;
-          bool valid = key < ti.nkeys;
-          if (ti.draft) valid = valid && draft_visible(p, sm.anc, rb * p.rows_per_unit + rl, ti.key0 + key);
-          s[j][e] = valid ? s[j][e] * qs : -INFINITY;
-          mx[e >> 1] = fmaxf(mx[e >> 1], s[j][e]);
+          for (int e = 0; e < 4; ++e) {
+            s[j][e] *= qs;
+            mx[e >> 1] = fmaxf(mx[e >> 1], s[j][e]);
+          }
+      } else {
+#pragma unroll
+        for (int j = 0; j < CF::kNT; ++j) {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int key = kw0 + j * 8 + 2 * q4 + (e & 1);
+            const int rl = rl0 + (e >> 1) * 8;
+            bool valid = key < ti.nkeys;
+            if (ti.draft) valid = valid && draft_visible(p, sm.anc, rb * p.rows_per_unit + rl, ti.key0 + key);
+            s[j][e] = valid ? s[j][e] * qs : -INFINITY;
+            mx[e >> 1] = fmaxf(mx[e >> 1], s[j][e]);
+          }
         }
       }
       float alpha[2], m_use[2];
@@ -422,15 +476,55 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
           pa[2] = pack_bf16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
           pa[3] = pack_bf16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
         }
-        const int key = kw0 + kk * 16 + ((lmat & 1) << 3) + lrow;
+        if constexpr (CF::kF8) {
+          // B fragments from key rows kb, kb + 1 (b0) and kb + 8, kb + 9 (b1), dims 16g .. 16g + 15:
+          // byte (or half-word) permutes pair the two rows' values of one dim, which lands in n8
+          // tile nd = dim - 16g at column g.  Rows past the tile's valid keys read as zero.
+          const int kb = kw0 + kk * 16 + 2 * q4;
+          const int rows[4] = {kb, kb + 1, kb + 8, kb + 9};
+          if (f16t) {
+            uint4 w[4];
 #pragma unroll
-        for (int ndp = 0; ndp < 8; ++ndp) {
-          uint32_t b0, b1, b2, b3;
-          ldmatrix_x4_trans(vbase + tile_off(key, 2 * ndp + (lmat >> 1)), b0, b1, b2, b3);
-          if constexpr (CF::kF8) {
-            mma_f16_16816(o[2 * ndp], pa, b0, b1);
-            mma_f16_16816(o[2 * ndp + 1], pa, b2, b3);
+            for (int r = 0; r < 4; ++r) {
+              w[r] = lds128(vbase + code_off(rows[r], g));
+              if (rows[r] >= ti.nkeys) w[r] = make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {  // dims 16g + 4t .. 4t + 3 -> tiles 4t .. 4t + 3
+              const uint2 ab0 = e4m3x4_to_f16x4(__byte_perm(word(w[0], t), word(w[1], t), 0x5140));
+              const uint2 ab1 = e4m3x4_to_f16x4(__byte_perm(word(w[0], t), word(w[1], t), 0x7362));
+              const uint2 cd0 = e4m3x4_to_f16x4(__byte_perm(word(w[2], t), word(w[3], t), 0x5140));
+              const uint2 cd1 = e4m3x4_to_f16x4(__byte_perm(word(w[2], t), word(w[3], t), 0x7362));
+              mma_f16_16816(o[4 * t], pa, ab0.x, cd0.x);
+              mma_f16_16816(o[4 * t + 1], pa, ab0.y, cd0.y);
+              mma_f16_16816(o[4 * t + 2], pa, ab1.x, cd1.x);
+              mma_f16_16816(o[4 * t + 3], pa, ab1.y, cd1.y);
+            }
           } else {
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {  // dims 16g + 8hh .. + 7 -> tiles 8hh .. 8hh + 7
+              uint4 w[4];
+#pragma unroll
+              for (int r = 0; r < 4; ++r) {
+                w[r] = lds128(vbase + tile_off(rows[r], 2 * g + hh));
+                if (rows[r] >= ti.nkeys) w[r] = make_uint4(0u, 0u, 0u, 0u);
+              }
+#pragma unroll
+              for (int t = 0; t < 4; ++t) {  // word t: dims 16g + 8hh + 2t, +1 -> tiles 8hh + 2t, +1
+                const uint32_t ab = word(w[0], t), bb = word(w[1], t), cb = word(w[2], t), db = word(w[3], t);
+                mma_f16_16816(o[8 * hh + 2 * t], pa, bf16x2_to_f16x2(__byte_perm(ab, bb, 0x5410)),
+                              bf16x2_to_f16x2(__byte_perm(cb, db, 0x5410)));
+                mma_f16_16816(o[8 * hh + 2 * t + 1], pa, bf16x2_to_f16x2(__byte_perm(ab, bb, 0x7632)),
+                              bf16x2_to_f16x2(__byte_perm(cb, db, 0x7632)));
+              }
+            }
+          }
+        } else {
+          const int key = kw0 + kk * 16 + ((lmat & 1) << 3) + lrow;
+#pragma unroll
+          for (int ndp = 0; ndp < 8; ++ndp) {
+            uint32_t b0, b1, b2, b3;
+            ldmatrix_x4_trans(vbase + tile_off(key, 2 * ndp + (lmat >> 1)), b0, b1, b2, b3);
             mma_bf16_16816(o[2 * ndp], pa, b0, b1);
             mma_bf16_16816(o[2 * ndp + 1], pa, b2, b3);
           }

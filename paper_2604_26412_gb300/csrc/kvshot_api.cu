@@ -53,8 +53,8 @@ bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// fp8 E4M3 target cache: one byte per element, whole 128-byte rows per box, no swizzle (the
-// m16n8k16 kernel expands each tile to the bf16 layout in shared memory).
+// fp8 E4M3 target cache: one byte per element, whole 128-byte rows per box, under the 128-byte
+// swizzle (the m16n8k16 kernel decodes the codes from shared memory straight into MMA fragments).
 bool encode_rows_fp8(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {
   auto fn = encode_fn();
   if (fn == nullptr) return false;
@@ -63,7 +63,7 @@ bool encode_rows_fp8(CUtensorMap* map, const void* base, uint64_t rows, uint32_t
   const cuuint32_t box[2] = {static_cast<cuuint32_t>(kHeadDim), box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -191,7 +191,7 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   //    shared memory into tensor memory, is faster (1.5x at 48 rows, 3-4x for
   //    whole-tree stacks of 128-256 rows).
   const bool tc_ok = G <= 128 && 128 % G == 0;
-  const bool fp8 = d->flags & KVSHOT_TARGET_FP8;  // only the m16n8k16 kernel expands fp8 tiles
+  const bool fp8 = d->flags & KVSHOT_TARGET_FP8;  // only the m16n8k16 kernel decodes fp8 tiles
   const Kernel automatic = (rows > 16 && tc_ok && !fp8) ? Kernel::kTensorMemory : Kernel::kMma;
   pl->kernel = force_cc ? Kernel::kCudaCore : force_tc ? Kernel::kTensorMemory
                                            : force_mma ? Kernel::kMma : automatic;

@@ -499,7 +499,7 @@ __device__ __forceinline__ void run_producer(const AttnParams& p, const TensorMa
         }
       } else if (p.paged) {
         // bf16: boxes of 64 dims per half; fp8 (p.fp8): one box of whole 128-byte rows, into the
-        // upper half of the tile (the lanes of half 1 skip), expanded there by the consumers.
+        // upper half of the tile (the lanes of half 1 skip), decoded from there by the consumers.
         const int br = p.box_rows;
         const int nbox = (nkeys + br - 1) / br;
         if (lane == 0) mbar_arrive_expect_tx(full_bar, nbox * br * 128 * (p.fp8 ? 2 : 4));
