@@ -112,6 +112,14 @@ ATTN_SOURCES = ("attn_cc.cu", "attn_mma.cu", "attn_tc.cu", "kvshot_api.cu", "kvs
                 "kvshot_internal.h", "kvshot_tcgen05.cuh", "merge_append.cu")
 
 
+# The sources each attention kernel's launches depend on: its own file, the shared producer/cursor
+# header, the host planner that sizes its grid, and the merge kernel.  A traffic record names the set
+# its hash covers, so an edit to one kernel leaves the other's record valid.
+MMA_SOURCES = ("attn_mma.cu", "kvshot_api.cu", "kvshot_attn_common.cuh", "kvshot_internal.h", "merge_append.cu")
+TC_SOURCES = ("attn_tc.cu", "kvshot_tcgen05.cuh", "kvshot_api.cu", "kvshot_attn_common.cuh", "kvshot_internal.h",
+              "merge_append.cu")
+
+
 # Sources of the gated-delta fusion call.
 FUSION_SOURCES = ("gated_delta.cu", "kvshot_slab_gemm.cuh", "kvshot_attn_common.cuh", "kvshot_internal.h", "kvshot_tcgen05.cuh")
 
@@ -125,9 +133,10 @@ def kernel_source_hash(sources=ATTN_SOURCES):
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload, mode, kernel_hash):
+def recorded_traffic(workload, mode, sources=ATTN_SOURCES):
     """DRAM bytes per call (key "w<workload>-<mode>", or "fusion-hybrid_tree") from a committed ncu
-    summary, if it is for the current kernel sources; else None."""
+    summary, if it is for the current kernel sources; else None.  The record's "sources" (default:
+    `sources`) are the files its "kernel_hash" covers."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
@@ -136,7 +145,7 @@ def recorded_traffic(workload, mode, kernel_hash):
         return None
     key = f"w{workload}-{mode}" if workload is not None else mode
     e = rec.get(key)
-    if not e or e.get("kernel_hash") != kernel_hash:
+    if not e or e.get("kernel_hash") != kernel_source_hash(tuple(e.get("sources", sources))):
         return None
     return e.get("dram_bytes_per_call")
 
@@ -376,7 +385,7 @@ def run_ours(args, world, rank, local):
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     khash = kernel_source_hash()
-    traffic = recorded_traffic(args.workload, args.mode + ("-fp8" if fp8 else ""), khash)
+    traffic = recorded_traffic(args.workload, args.mode + ("-fp8" if fp8 else ""))
     rows_per_head = spec.hq // spec.hkv * max(levels)
     roofline = {
         "bound": "hbm",
@@ -554,7 +563,7 @@ def run_fusion(args, world, rank, local):
         "unit": "GB/s",
         "frac": round(achieved / hbm_peak, 4),
         "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6.8 TB/s",
-        "traffic": recorded_traffic(None, "fusion-hybrid_tree", kernel_source_hash(FUSION_SOURCES)),
+        "traffic": recorded_traffic(None, "fusion-hybrid_tree", FUSION_SOURCES),
         "algorithmic_bytes_per_call": int(statistics.mean(call_bytes)),
         "call_us": round(statistics.mean(call_ms) * 1e3, 2),
         "per_level_us": [round(x * 1e3, 2) for x in call_ms],

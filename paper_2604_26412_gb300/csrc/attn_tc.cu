@@ -327,10 +327,20 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         }
         const uint64_t vis = v64 >> col0;  // bit j = column col0 + j
         float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        // Dense rows skip the per-key mask on a full prefix tile (every key is visible): +6% on the
+        // 128-row whole-tree stacks; spread rows (half the columns) measured ~2-4% slower with it.
+        if (!kSpread && valid && !ti.draft && ti.nkeys >= kTileKeys) {
 #pragma unroll
-        for (int j = 0; j < kCols; ++j) {
-          pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * qscale : -INFINITY;
-          mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
+          for (int j = 0; j < kCols; ++j) {
+            pr[j] = __uint_as_float(sv[j]) * qscale;
+            mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < kCols; ++j) {
+            pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * qscale : -INFINITY;
+            mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
+          }
         }
         float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
         if constexpr (kSpread) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
