@@ -42,3 +42,32 @@ def test_flops_and_fusion_bytes():
 def test_whole_job_rate_counts_every_rank_against_the_slowest():
     assert replicas.whole_job_rate(100, steps=10, world=1, max_ms=2.0) == 500_000.0
     assert replicas.whole_job_rate(100, steps=10, world=4, max_ms=2.0) == 2_000_000.0
+
+
+def test_traffic_records_are_well_formed(tmp_path, monkeypatch):
+    """Every committed traffic record has positive DRAM bytes and names an existing profile summary
+    and existing kernel sources; the lookup uses a record only while its sources hash to its
+    kernel_hash."""
+    import json
+    import os
+    rec = json.load(open(os.path.join(bench.ROOT, "profiles", "traffic.json")))
+    csrc = os.path.join(bench.ROOT, "paper_2604_26412_gb300", "csrc")
+    assert rec, "no traffic records"
+    for key, e in rec.items():
+        assert e["dram_bytes_per_call"] > 0, key
+        assert os.path.exists(os.path.join(bench.ROOT, e["profile"])), key
+        assert len(e["kernel_hash"]) == 16, key
+        for name in e.get("sources", ()):
+            assert os.path.exists(os.path.join(csrc, name)), (key, name)
+    # a record is used only while its sources hash to its kernel_hash
+    fake_root = tmp_path
+    os.makedirs(fake_root / "profiles")
+    os.symlink(os.path.join(bench.ROOT, "paper_2604_26412_gb300"), fake_root / "paper_2604_26412_gb300")
+    good = {"kernel_hash": bench.kernel_source_hash(bench.MMA_SOURCES), "sources": list(bench.MMA_SOURCES),
+            "dram_bytes_per_call": 123.0, "how": "", "profile": ""}
+    stale = dict(good, kernel_hash="0" * 16)
+    (fake_root / "profiles" / "traffic.json").write_text(json.dumps({"w5-per_depth": good, "w4-per_depth": stale}))
+    monkeypatch.setattr(bench, "ROOT", str(fake_root))
+    assert bench.recorded_traffic(5, "per_depth") == 123.0
+    assert bench.recorded_traffic(4, "per_depth") is None
+    assert bench.recorded_traffic(3, "per_depth") is None
