@@ -26,6 +26,7 @@ import io
 import json
 import math
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -124,12 +125,23 @@ TC_SOURCES = ("attn_tc.cu", "kvshot_tcgen05.cuh", "kvshot_api.cu", "kvshot_attn_
 FUSION_SOURCES = ("gated_delta.cu", "kvshot_slab_gemm.cuh", "kvshot_attn_common.cuh", "kvshot_internal.h", "kvshot_tcgen05.cuh")
 
 
+# Comments, string and character literals of C/C++/CUDA source, in the order a compiler reads them.
+_CXX_TOKENS = re.compile(r'//[^\n]*|/\*.*?\*/|"(?:\\.|[^"\\\n])*"|\'(?:\\.|[^\'\\\n])*\'', re.S)
+
+
+def code_only(text: str) -> str:
+    """The source with its comments removed and its whitespace collapsed (literals kept as written)."""
+    return " ".join(_CXX_TOKENS.sub(lambda m: " " if m.group(0)[0] == "/" else m.group(0), text).split())
+
+
 def kernel_source_hash(sources=ATTN_SOURCES):
+    """Hash of the code (comments and whitespace ignored) of the given csrc files: a traffic record
+    stays valid across edits that cannot change the kernels' DRAM traffic."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2604_26412_gb300", "csrc")
     for name in sources:
-        with open(os.path.join(csrc, name), "rb") as f:
-            h.update(name.encode() + f.read())
+        with open(os.path.join(csrc, name), encoding="utf-8") as f:
+            h.update(name.encode() + b"\0" + code_only(f.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -16,8 +16,8 @@
 // f16 with the cache's power-of-two scales folded into the score scale and
 // into P.  Fragment layouts of that variant: a lane's 16-byte load of one key
 // row feeds four k-steps of S = Q K^T, so the head dimensions of q are taken
-// in the same permuted order (k-step 4h + s, pair position 2 q4 -> dims
-// 16 (2 q4 + h) + 4 s + {0, 1}, position 8 + 2 q4 -> + {2, 3}); for O += P V a
+// in the same permuted order (k-step 4 kh + s, pair position 2 q4 -> dims
+// 16 (2 q4 + kh) + 4 s + {0, 1}, position 8 + 2 q4 -> + {2, 3}); for O += P V a
 // lane pairs the same 16 dims of two key rows with byte permutes, so the
 // output columns are permuted too (n8 tile nd, column n -> dim 16 n + nd) and
 // the write-out undoes it.  Draft tiles (bf16) are read into the same layouts
@@ -306,7 +306,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
             p.q + ((static_cast<size_t>(cu.c) * p.Nq + nl) * p.hq + h * p.G + gh) * kHeadDim);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          if constexpr (CF::kF8) {  // f16, k-step 4h + s on dims 16 (2 q4 + h) + 4 s + {0..3}
+          if constexpr (CF::kF8) {  // f16, k-step 4 kh + s on dims 16 (2 q4 + kh) + 4 s + {0..3}
             const int w = 8 * (2 * q4 + (kk >> 2)) + 2 * (kk & 3);
             qa[kk][i] = ok ? bf16x2_to_f16x2(src[w]) : 0u;
             qa[kk][2 + i] = ok ? bf16x2_to_f16x2(src[w + 1]) : 0u;

@@ -71,3 +71,19 @@ def test_traffic_records_are_well_formed(tmp_path, monkeypatch):
     assert bench.recorded_traffic(5, "per_depth") == 123.0
     assert bench.recorded_traffic(4, "per_depth") is None
     assert bench.recorded_traffic(3, "per_depth") is None
+
+
+def test_source_hash_ignores_comments_not_code(tmp_path, monkeypatch):
+    import os
+    csrc = tmp_path / "paper_2604_26412_gb300" / "csrc"
+    os.makedirs(csrc)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    base = 'int f(int a) { return a / 2; }  // halve\nconst char* s = "x // y";\n'
+    (csrc / "k.cu").write_text(base)
+    h0 = bench.kernel_source_hash(("k.cu",))
+    (csrc / "k.cu").write_text("/* header */\n" + base.replace("// halve", "// half of a, it's exact") + "\n\n")
+    assert bench.kernel_source_hash(("k.cu",)) == h0            # comments and blank lines only
+    (csrc / "k.cu").write_text(base.replace("a / 2", "a / 3"))
+    assert bench.kernel_source_hash(("k.cu",)) != h0            # code
+    (csrc / "k.cu").write_text(base.replace('"x // y"', '"x // z"'))
+    assert bench.kernel_source_hash(("k.cu",)) != h0            # a string literal is code
