@@ -306,6 +306,123 @@ class OracleSample:
 
 # ---------------------------------------------------------------- our arm
 
+def attn_config(spec: wl.Spec, args, world: int, bytes_per_call: float) -> dict:
+    """The workload block of the JSON line; the reference arm prints the same block."""
+    paged = spec.paged
+    fp8 = args.kv_dtype == "fp8"
+    return {
+        "workload": spec.name,
+        "mode": args.mode,
+        "num_seqs": spec.num_seqs,
+        "reused_layers": spec.layers,
+        "num_caches": spec.num_caches,
+        "prefix_lens": "ragged U[512,8192]" if args.workload == 4 else spec.seq_lens[0],
+        "draft_levels": list(spec.levels),
+        "tree": spec.tree,
+        "layout": f"paged P={spec.page_size}" if paged else "contiguous",
+        "target_cache": "fp8 e4m3" if fp8 else "bf16",
+        "append": "QK-norm + RoPE" if args.qk_norm else "RoPE",
+        "gqa": f"{spec.hq}/{spec.hkv}",
+        "head_dim": spec.head_dim,
+        "tokens_per_step": spec.num_seqs * spec.n_nodes,
+        "l2": "inputs larger than L2 (no flush)" if bytes_per_call > 2 * 129e6
+              else "inputs smaller than L2 (not flushed: latency-bound workload)",
+        "parallelism": f"replicas x{world}",
+    }
+
+
+def mode_levels(spec: wl.Spec, mode: str):
+    """Query nodes per draft-attention call of one step: one call per depth, or one for the whole tree."""
+    return list(spec.levels) if mode == "per_depth" else [spec.n_nodes]
+
+
+def roofline_bytes(spec: wl.Spec, levels, paged: bool, fp8: bool):
+    n0s = np.cumsum([0] + list(levels)[:-1]).tolist()
+    return [algorithmic_bytes(spec, n0s[i] + levels[i], levels[i], paged, 1 if fp8 else 2) for i in range(len(levels))]
+
+
+def call_roofline(step, inp, spec: wl.Spec, stream, ms_per_step: float, hbm_peak: float, peak_src: str, traffic=None,
+                  target_elem: int = 2) -> dict:
+    """Live roofline of the draft-attention calls of one step (attention + merge kernels): CUDA events
+    around every call on the launching stream, the stream kept busy by a sleep kernel while the host
+    enqueues them; achieved = algorithmic bytes / mean call time."""
+    from paper_2604_26412_gb300 import kvshot
+    levels = step.levels
+    n0s = np.cumsum([0] + levels[:-1]).tolist()
+    paged = inp.page_table is not None
+    reps = max(3, min(50, int(2000 / max(ms_per_step, 1e-3) / len(levels))))
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in levels]
+          for _ in range(reps)]
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(2e7))  # keep the GPU busy while the host enqueues the calls
+        for r in range(reps):
+            for i in range(len(levels)):
+                ev[r][i][0].record(stream)
+                kvshot.draft_attn(step.descs[i], step.q_rot[i], step.target_k, step.target_v, inp.page_table,
+                                  inp.seq_lens, step.draft_k, step.draft_v, step.parents[i], step.out[i], step.lse[i],
+                                  stream)
+                ev[r][i][1].record(stream)
+    torch.cuda.synchronize()
+    if step.error_code() != 0:
+        raise RuntimeError(f"device error {step.error_code()}")
+    call_ms = [statistics.mean(ev[r][i][0].elapsed_time(ev[r][i][1]) for r in range(reps)) for i in range(len(levels))]
+    call_bytes = [algorithmic_bytes(spec, n0s[i] + levels[i], levels[i], paged, target_elem) for i in range(len(levels))]
+    call_flops = [algorithmic_flops(spec, n0s[i] + levels[i], levels[i]) for i in range(len(levels))]
+    achieved_gbs = sum(call_bytes) / (sum(call_ms) / 1e3) / 1e9
+    achieved_tflops = sum(call_flops) / (sum(call_ms) / 1e3) / 1e12
+    G = spec.hq // spec.hkv
+    kernels = sorted({"tcgen05" if G * lv > 16 and 128 % G == 0 and target_elem == 2 else "m16n8k16"
+                      for lv in levels})
+    return {
+        "bound": "hbm",
+        "kernel": "kvshot_draft_attn (attention + merge kernels)",
+        "attention_kernels": kernels,
+        "achieved": round(achieved_gbs, 1),
+        "peak": hbm_peak,
+        "unit": "GB/s",
+        "frac": round(achieved_gbs / hbm_peak, 4),
+        "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6.8 TB/s",
+        "traffic": traffic,
+        "algorithmic_bytes_per_call": int(statistics.mean(call_bytes)),
+        "call_us": round(statistics.mean(call_ms) * 1e3, 2),
+        "per_level_us": [round(x * 1e3, 2) for x in call_ms],
+        "achieved_tflops": round(achieved_tflops, 2),
+        "max_rows_per_kv_head": G * max(levels),
+        "calls_timed": reps * len(levels),
+        "kernel_hash": kernel_source_hash(),
+    }
+
+
+def gate_roofline(workload: int, args, dev, hbm_peak: float, peak_src: str) -> dict:
+    """Live roofline of another workload's draft-attention calls (per depth, default kernels), measured
+    in the same process after a few untimed steps."""
+    from paper_2604_26412_gb300.step import DraftStep
+    spec = wl.config(workload, seed=args.seed)
+    inp = wl.make_inputs(spec, dev, seed=args.seed)
+    step = DraftStep(inp, mode="per_depth")
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            step.run()
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        s0.record(stream)
+        for _ in range(5):
+            step.run()
+        s1.record(stream)
+    torch.cuda.synchronize()
+    r = call_roofline(step, inp, spec, stream, s0.elapsed_time(s1) / 5, hbm_peak, peak_src,
+                      traffic=recorded_traffic(workload, "per_depth"))
+    out = {"workload": spec.name, "mode": "per_depth"}
+    out.update({k: r[k] for k in ("frac", "achieved", "unit", "call_us", "per_level_us", "traffic",
+                                  "algorithmic_bytes_per_call", "attention_kernels", "calls_timed")})
+    del step, inp
+    torch.cuda.empty_cache()
+    return out
+
+
+
 def run_ours(args, world, rank, local):
     from paper_2604_26412_gb300 import kvshot
     from paper_2604_26412_gb300.step import DraftStep
@@ -373,53 +490,25 @@ def run_ours(args, world, rank, local):
     value = replicas.whole_job_rate(tokens_per_step, args.steps, world, ms_total)
 
     # ---- live roofline of the draft-attention call (attention + merge kernels), per level
-    levels = step.levels
-    n0s = np.cumsum([0] + levels[:-1]).tolist()
-    reps = max(3, min(50, int(2000 / max(ms_per_step, 1e-3) / len(levels))))
-    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in levels]
-          for _ in range(reps)]
-    with torch.cuda.stream(stream):
-        torch.cuda._sleep(int(2e7))  # keep the GPU busy while the host enqueues the calls
-        for r in range(reps):
-            for i in range(len(levels)):
-                ev[r][i][0].record(stream)
-                kvshot.draft_attn(step.descs[i], step.q_rot[i], step.target_k, step.target_v, inp.page_table,
-                                  inp.seq_lens, step.draft_k, step.draft_v, step.parents[i], step.out[i], step.lse[i],
-                                  stream)
-                ev[r][i][1].record(stream)
-    torch.cuda.synchronize()
-    call_ms = [statistics.mean(ev[r][i][0].elapsed_time(ev[r][i][1]) for r in range(reps)) for i in range(len(levels))]
-    call_bytes = [algorithmic_bytes(spec, n0s[i] + levels[i], levels[i], paged, 1 if fp8 else 2)
-                  for i in range(len(levels))]
-    call_flops = [algorithmic_flops(spec, n0s[i] + levels[i], levels[i]) for i in range(len(levels))]
-    achieved_gbs = sum(call_bytes) / (sum(call_ms) / 1e3) / 1e9
-    achieved_tflops = sum(call_flops) / (sum(call_ms) / 1e3) / 1e12
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
-    khash = kernel_source_hash()
-    traffic = recorded_traffic(args.workload, args.mode + ("-fp8" if fp8 else ""))
-    rows_per_head = spec.hq // spec.hkv * max(levels)
-    roofline = {
-        "bound": "hbm",
-        "kernel": "kvshot_draft_attn (attention + merge kernels)",
-        "achieved": round(achieved_gbs, 1),
-        "peak": hbm_peak,
-        "unit": "GB/s",
-        "frac": round(achieved_gbs / hbm_peak, 4),
-        "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6.8 TB/s",
-        "traffic": traffic,
-        "algorithmic_bytes_per_call": int(statistics.mean(call_bytes)),
-        "call_us": round(statistics.mean(call_ms) * 1e3, 2),
-        "per_level_us": [round(x * 1e3, 2) for x in call_ms],
-        "achieved_tflops": round(achieved_tflops, 2),
-        "max_rows_per_kv_head": rows_per_head,
-        "kernel_hash": khash,
-    }
+    roofline = call_roofline(step, inp, spec, stream, ms_per_step, hbm_peak, peak_src,
+                             traffic=recorded_traffic(args.workload, args.mode + ("-fp8" if fp8 else "")),
+                             target_elem=1 if fp8 else 2)
+    gates = None
+    if args.workload == 5 and args.mode == "per_depth" and not fp8 and flags == 0 and not args.qk_norm \
+            and not args.max_prefix and not args.page_size:
+        # The other long-prefix workloads, per depth, measured the same way in the same process.
+        gate_clocks = ClockSampler(local)
+        gate_clocks.start()
+        gates = {f"w{w}": gate_roofline(w, args, dev, hbm_peak, peak_src) for w in (3, 4)}
+        gates["clocks"] = gate_clocks.stop()
+        gates["w5"] = {k: roofline[k] for k in ("frac", "achieved", "call_us")}
 
     # ---- end to end through the C ABI with host buffers (pinned), copies in the timed region
     e2e = run_e2e(args, step, inp, stream, world)
 
-    gpu_launches = 3 * len(levels) * args.steps
+    gpu_launches = 3 * len(step.levels) * args.steps
     result = {
         "metric": METRIC,
         "value": round(value, 1),
@@ -434,31 +523,15 @@ def run_ours(args, world, rank, local):
         "dtype": "bf16 (target K/V fp8 e4m3)" if fp8 else "bf16",
         "data": "synthetic (seeded N(0,1) K/V, N(0,1)/sqrt(128) q; shapes of the paper's Qwen3-8B runs)"
                 + (f"; target cache as e4m3 codes x 2^{wl.FP8_K_EXP} (K), 2^{wl.FP8_V_EXP} (V)" if fp8 else ""),
-        "config": {
-            "workload": spec.name,
-            "mode": args.mode,
-            "num_seqs": spec.num_seqs,
-            "reused_layers": spec.layers,
-            "num_caches": spec.num_caches,
-            "prefix_lens": "ragged U[512,8192]" if args.workload == 4 else spec.seq_lens[0],
-            "draft_levels": list(spec.levels),
-            "tree": spec.tree,
-            "layout": f"paged P={spec.page_size}" if paged else "contiguous",
-            "target_cache": "fp8 e4m3" if fp8 else "bf16",
-            "append": "QK-norm + RoPE" if args.qk_norm else "RoPE",
-            "gqa": f"{spec.hq}/{spec.hkv}",
-            "head_dim": spec.head_dim,
-            "tokens_per_step": tokens_per_step,
-            "cuda_graph": graph is not None,
-            "l2": "inputs larger than L2 (no flush)" if sum(call_bytes) / len(call_bytes) > 2 * 129e6
-                  else "inputs smaller than L2 (not flushed: latency-bound workload)",
-            "parallelism": f"replicas x{world}",
-        },
+        "config": attn_config(spec, args, world, sum(roofline_bytes(spec, step.levels, paged, fp8)) / len(step.levels)),
+        "cuda_graph": graph is not None,
         "roofline": roofline,
         "e2e": e2e,
         "clocks": clock_info,
         "gpu_launches": gpu_launches,
     }
+    if gates is not None:
+        result["gates"] = gates
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         samp = OracleSample(spec, args.mode, args.seed)
         v, desc, _ = samp.timed(args.cpu_sample_seconds)
@@ -923,7 +996,10 @@ def run_reference(args):
         "vs_baseline": None,
         "dtype": "f64",
         "data": "synthetic (seeded; same shapes as the GPU arm)",
-        "config": {"workload": spec.name, "mode": args.mode, "parallelism": "host cores"},
+        "config": attn_config(spec, args, args.gpus,
+                              sum(roofline_bytes(spec, mode_levels(spec, args.mode), spec.paged,
+                                                 args.kv_dtype == "fp8")) / len(mode_levels(spec, args.mode))),
+        "host_parallelism": f"fp64 oracle on {samp.cores} host cores (rank 0 only)",
         "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": samp.cores, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

@@ -21,6 +21,12 @@
 // written, so QK^T runs ahead of the softmax.  O_w is rescaled in
 // TMEM only when a row's running max grows by more than 2^8 (lazy rescale).
 // Rows of the 128-row MMA that hold no stacked row carry no output.
+// K and V tiles are staged in the grouped layout (kGroupBytes): one TMA box
+// brings a whole page of up to 64 tokens with both 64-dim halves, so a tile of
+// 16-token pages takes 4 boxes per tensor instead of 8.  Ring depths (4 K,
+// 5 V, 2 P buffers) were measured on GB300: the bytes in flight per SM that
+// the K and V rings allow bound how fast one CTA streams, and a third P buffer
+// gained nothing.
 #include "kvshot_attn_common.cuh"
 #include "kvshot_tcgen05.cuh"
 
@@ -30,11 +36,11 @@ namespace {
 using namespace dev;
 using namespace tc;
 
-constexpr int kNK = 3;                     // K tiles in flight (freed when QK^T completes)
+constexpr int kNK = 4;                     // K tiles in flight (freed when QK^T completes)
 constexpr int kNV = 5;                     // V tiles in flight (freed when P.V completes)
 constexpr int kKVBytes = kKVTileBytes;     // one K or V tile
 constexpr int kNS = 4;                     // S buffers in TMEM: QK^T may run up to 4 tiles ahead of P.V
-constexpr int kNP = 3;                     // P buffers in shared memory
+constexpr int kNP = 2;                     // P buffers in shared memory (buffer w: warpgroup w's tiles)
 constexpr int kThreads = 12 * 32;
 constexpr int kProducerWarp = 10;          // K and V loads of even tiles
 constexpr int kProducerVWarp = 9;          // K and V loads of odd tiles, q blocks
@@ -47,6 +53,14 @@ constexpr uint32_t kTmemCols = 512;        // S0..S3 [0,256), O0 [256,384), O1 [
 constexpr uint32_t kTmemO = kNS * kTileKeys;
 constexpr int kMiscInts = 12;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max grows by > 256x
+
+// Byte offset of 16-byte chunk `ch` (dims 8ch..8ch+7) of key r in a K or V
+// tile of either layout (128-byte swizzle: chunk index XOR row index mod 8).
+__device__ __forceinline__ uint32_t tile_off_tc(int r, int ch, bool grouped) {
+  const uint32_t sw = static_cast<uint32_t>(((ch & 7) ^ (r & 7)) << 4);
+  if (grouped) return static_cast<uint32_t>((r >> 3) * kGroupBytes + (ch >> 3) * kGroupHalfBytes + (r & 7) * 128) + sw;
+  return static_cast<uint32_t>((ch >> 3) * kHalfBytes + r * 128) + sw;
+}
 
 // ------------------------------------------------------------ shared memory
 
@@ -147,10 +161,14 @@ __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, 
     tc_fence_after();
     const uint32_t qbase = smem_addr(sm.qbuf);
     const uint32_t kbase = smem_addr(sm.kring + static_cast<size_t>(t % kNK) * kKVBytes);
+    // K tile: 8-key groups (the MMA's N direction) kGroupBytes apart and the dims 64..127 half
+    // kGroupHalfBytes on (grouped layout), or 1 KB and kHalfBytes (halves layout).
+    const bool grouped = ti.draft || p.prefix_grouped;
+    const uint32_t half_off = grouped ? kGroupHalfBytes : kHalfBytes, group_off = grouped ? kGroupBytes : 1024;
 #pragma unroll
     for (int ks = 0; ks < kHeadDim / 16; ++ks) {
       const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
-      const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * kHalfBytes + (ks & 3) * 32, 16, 1024);
+      const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * half_off + (ks & 3) * 32, 16, group_off);
       tc_mma(tmem + (t % kNS) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
     }
     tc_commit(smem_addr(&sm.sfull[t % kNS]));
@@ -186,11 +204,13 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
     const uint32_t pbase = smem_addr(sm.pbuf + (t % kNP) * kPBufBytes);
     const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(t % kNV) * kKVBytes);
     const uint32_t o = tmem + kTmemO + 128 * (t & 1);
+    const bool grouped = ti.draft || p.prefix_grouped;
+    const uint32_t half_off = grouped ? kGroupHalfBytes : kHalfBytes, group_off = grouped ? kGroupBytes : 1024;
 #pragma unroll
     for (int k16 = 0; k16 < kTileKeys / 16; ++k16) {  // 16-key steps of the tile
       const uint64_t a = smem_desc_sw128(pbase + k16 * 32, 16, 1024);
-      // V tile is MN-major: 64-dim halves 8 KB apart (leading), 8-key groups 1 KB apart (stride).
-      const uint64_t bd = smem_desc_sw128(vbase + k16 * 2048, kHalfBytes, 1024);
+      // V tile is MN-major: 64-dim halves `half_off` apart (leading), 8-key groups `group_off` apart (stride).
+      const uint64_t bd = smem_desc_sw128(vbase + k16 * 2 * group_off, half_off, group_off);
       tc_mma(o, a, bd, idesc, (first && k16 == 0) ? 0u : 1u);
     }
     tc_commit(smem_addr(&sm.vempty[t % kNV]));
@@ -396,7 +416,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         const int nz = (kTileKeys - ti.nkeys) * 16;
         for (int i = wtid; i < nz; i += kSoftmaxThreads / 2) {
           const int key = ti.nkeys + (i >> 4), ch = i & 15;
-          *reinterpret_cast<uint4*>(vptr + tile_off(key, ch)) = make_uint4(0, 0, 0, 0);
+          *reinterpret_cast<uint4*>(vptr + tile_off_tc(key, ch, ti.draft || p.prefix_grouped)) = make_uint4(0, 0, 0, 0);
         }
       }
       fence_proxy_async_smem();
@@ -506,41 +526,62 @@ struct FastDiv {
   }
 };
 
-// TMA boxes of one K (or V) tile: `nbox` (<= 8) boxes of `br` rows in each
-// 64-dim half; lanes l and l + 16 (hf = l & 1, i = (l & 15) >> 1) own box i of
-// half hf, whose first row in the tile's tensor map (target or draft) is y.  h is the unit's KV
+// TMA boxes of one K (or V) tile; this lane's box is i = lane & 15 (at most
+// 8 per tensor).  Grouped layout (draft tiles, and prefix tiles when
+// p.prefix_grouped): a box holds whole 8-key groups with both 64-dim halves
+// (a page of P <= 64 tokens, a 64-token slice of a larger page or of the
+// contiguous cache, or 8 draft slots); halves layout (a contiguous cache whose
+// l_cap is not a multiple of 8): one box per 64-dim half.  h is the unit's KV
 // head, `pages` the cache's pages in use.  Warp-wide.
 struct TileBoxes {
-  bool draft;
-  int y, nbox, br;
+  bool draft, grouped;
+  int nbox;        // boxes per tensor
+  int x, y;        // this lane's box: map coordinates (x: halves layout only)
+  uint32_t off;    // this lane's box: byte offset in the tile
+  uint32_t bytes;  // bytes of all of one tensor's boxes
 };
 
 __device__ __forceinline__ TileBoxes tile_boxes(const AttnParams& p, const Cursor& cu, PageWindow& win, int lane,
                                                 int h, int pages, const FastDiv& pdiv) {
   TileBoxes tb;
   tb.draft = cu.lt >= cu.pt;
+  tb.grouped = tb.draft || p.prefix_grouped;
+  tb.x = 0;
   const int key0 = (tb.draft ? cu.lt - cu.pt : cu.lt) * kTileKeys;
   const int nkeys = min(kTileKeys, (tb.draft ? p.N : cu.L) - key0);
-  const int i = (lane & 15) >> 1;
+  const int i = lane & 15;
   if (tb.draft) {
-    tb.br = kDraftBoxRows;
+    // 3-D map {64 dims, rows, 2 halves}: first row of the box.
     tb.nbox = (nkeys + kDraftBoxRows - 1) / kDraftBoxRows;
-    tb.y = (cu.c * p.hkv + h) * p.n_max + key0 + i * tb.br;
+    tb.y = (cu.c * p.hkv + h) * p.n_max + key0 + i * kDraftBoxRows;
+    tb.off = static_cast<uint32_t>(i) * kGroupBytes;
+    tb.bytes = static_cast<uint32_t>(tb.nbox) * kGroupBytes;
   } else if (p.paged) {
-    // Pages of P <= 64 rows: one box per page (P divides the tile); larger
-    // pages: one 64-row box inside the page.
+    // 4-D map {64 dims, 8 rows, 2 halves, row groups}: row group of the box.  Pages of
+    // P <= 64 tokens: one box per page (P divides the tile); larger pages: one 64-row box.
     const int P = p.page_size;
-    tb.br = p.box_rows;
-    tb.nbox = tb.br < kTileKeys ? pdiv.div(nkeys + P - 1) : 1;
+    const bool small_pages = P < kTileKeys;
+    tb.nbox = small_pages ? pdiv.div(nkeys + P - 1) : 1;
     const int pg0 = pdiv.div(key0);
-    const int npg = tb.br < P ? 1 : tb.nbox;
+    const int npg = small_pages ? tb.nbox : 1;
     win.cover(p, cu.c, pages, pg0, npg, lane);
-    const int pid = win.get(pg0 + (tb.br < P ? 0 : min(i, npg - 1)));
-    tb.y = (pid * p.hkv + h) * P + (tb.br < P ? key0 - pg0 * P : 0);
-  } else {
-    tb.br = kTileKeys;
+    const int pid = win.get(pg0 + (small_pages ? min(i, npg - 1) : 0));
+    tb.y = ((pid * p.hkv + h) * P + (small_pages ? 0 : key0 - pg0 * P)) >> 3;
+    const uint32_t box_bytes = small_pages ? static_cast<uint32_t>(P) * 256u : kKVTileBytes;
+    tb.off = static_cast<uint32_t>(i) * box_bytes;
+    tb.bytes = static_cast<uint32_t>(tb.nbox) * box_bytes;
+  } else if (p.prefix_grouped) {
     tb.nbox = 1;
+    tb.y = ((cu.c * p.hkv + h) * p.l_cap + key0) >> 3;
+    tb.off = 0;
+    tb.bytes = kKVTileBytes;
+  } else {
+    // 2-D map {128 dims, rows}, boxes {64 dims, 64 rows}: box i is half i.
+    tb.nbox = 2;
+    tb.x = i * 64;
     tb.y = (cu.c * p.hkv + h) * p.l_cap + key0;
+    tb.off = static_cast<uint32_t>(i) * kHalfBytes;
+    tb.bytes = kKVTileBytes;
   }
   return tb;
 }
@@ -623,9 +664,8 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
       wait_for_prerequisite_grid();
       waited = true;
     }
-    // Lanes 0..15 load the K boxes, lanes 16..31 the V boxes (half = lane & 1, row group = (lane & 15) >> 1).
-    const int kv = lane >> 4, hf = lane & 1, i = (lane & 15) >> 1;
-    const uint32_t tx = tb.nbox * tb.br * 128 * 2;  // bytes of one K (or V) tile's boxes
+    // Lanes 0..15 load the K boxes, lanes 16..31 the V boxes (box = lane & 15).
+    const int kv = lane >> 4, i = lane & 15;
     const int kslot = t % kNK, vslot = t % kNV;
     // A V slot is free once P.V of its previous tile completed, a K slot once QK^T of its previous tile
     // (t - kNK) completed.  Lane 0 waits for the K slot and lane 1 for the V slot together.
@@ -641,13 +681,14 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
       break;
     }
     const uint32_t full_bar = smem_addr(kv ? &sm.vfull[vslot] : &sm.kfull[kslot]);
-    if ((lane & 15) == 0) mbar_arrive_expect_tx(full_bar, tx);
+    if ((lane & 15) == 0) mbar_arrive_expect_tx(full_bar, tb.bytes);
     if (i < tb.nbox) {
       const uint32_t dst = smem_addr((kv ? sm.vring + static_cast<size_t>(vslot) * kKVBytes
                                          : sm.kring + static_cast<size_t>(kslot) * kKVBytes)) +
-                           hf * kHalfBytes + i * tb.br * 128;
-      const CUtensorMap* map = tb.draft ? (kv ? &maps.dv : &maps.dk) : (kv ? &maps.tv : &maps.tk);
-      tma_load_2d(dst, map, hf * 64, tb.y, full_bar, policy);
+                           tb.off;
+      if (tb.draft) tma_load_3d(dst, kv ? &maps.dv : &maps.dk, 0, tb.y, 0, full_bar, policy);
+      else if (tb.grouped) tma_load_4d_hint(dst, kv ? &maps.tv : &maps.tk, 0, 0, 0, tb.y, full_bar, policy);
+      else tma_load_2d(dst, kv ? &maps.tv : &maps.tk, tb.x, tb.y, full_bar, policy);
     }
     if (lane == 0) {
       sm.misc[8 + role] = t + 1;

@@ -67,9 +67,45 @@ bool encode_rows_fp8(CUtensorMap* map, const void* base, uint64_t rows, uint32_t
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Grouped views of a [rows, 128] bf16 matrix for the tensor-memory kernel (kGroupBytes in
+// kvshot_internal.h): a box lands as 8-row groups of 2 KB, each holding its rows' dims 0..63
+// (128-byte swizzled) and then dims 64..127.
+//  - 4-D {64 dims, 8 rows, 2 halves, rows / 8} (rows % 8 == 0), box {64, 8, 2, groups}: whole
+//    8-row groups from a row-group coordinate (pages and aligned cache slices);
+//  - 3-D {64 dims, rows, 2 halves}, box {64, 8, 2}: one group from any first row (draft slots).
+// The halves dimension's stride (128 B) is below the rows' (256 B): both views address every
+// element of the matrix exactly once.
+bool encode_rows_grouped(CUtensorMap* map, const void* base, uint64_t rows, uint32_t groups) {
+  auto fn = encode_fn();
+  if (fn == nullptr || rows % 8 != 0) return false;
+  const cuuint64_t dims[4] = {64, 8, 2, static_cast<cuuint64_t>(rows / 8)};
+  const cuuint64_t strides[3] = {256, 128, 2048};
+  const cuuint32_t box[4] = {64, 8, 2, groups};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_rows_group3(CUtensorMap* map, const void* base, uint64_t rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[3] = {64, static_cast<cuuint64_t>(rows), 2};
+  const cuuint64_t strides[2] = {256, 128};
+  const cuuint32_t box[3] = {64, 8, 2};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 constexpr int kMaxScaleExp = 64;
 
 enum class Kernel { kCudaCore, kMma, kTensorMemory };
+
+// Fixed cost, in 64-key tile times of one CTA, of splitting units across CTAs (piece epilogues
+// that stall the pipeline mid-stream, the merge kernel after the last CTA); measured on GB300.
+constexpr int64_t kSplitCostTiles = 15;
 
 }  // namespace
 
@@ -229,6 +265,15 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
     const int sms = sm_count();
     if (e != cudaSuccess || per_sm < 1 || sms < 1) return KVSHOT_ERR_CUDA;
     grid = sms * per_sm;
+    // Tensor-memory kernel: when every unit fits on a CTA of its own and the SMs that would stay
+    // idle would take fewer than kSplitCostTiles tiles off each CTA, give each unit its own CTA:
+    // no unit is split, so no piece epilogue runs mid-stream and the merge has nothing to do.
+    // (GB300, 128 units of 65 tiles, 16-token pages: 56.4 us per call on 128 CTAs against 59.9 us
+    // on 152; 128 units of 514 tiles stay faster split over all SMs.)
+    if (pl->kernel == Kernel::kTensorMemory && units <= grid) {
+      const int64_t unit_tiles = (static_cast<int64_t>(d->max_seq_len) + kTileKeys - 1) / kTileKeys + pl->draft_tiles;
+      if (unit_tiles * (grid - units) < kSplitCostTiles * static_cast<int64_t>(grid)) grid = static_cast<int>(units);
+    }
   }
   grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(grid, std::max<int64_t>(1, max_tiles))));
   pl->num_ctas = grid;
@@ -296,13 +341,26 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   const uint32_t tbox = paged ? static_cast<uint32_t>(std::min(d->page_size, kTileKeys)) : kTileKeys;
   const uint64_t drows = static_cast<uint64_t>(d->num_caches) * d->hkv * d->n_max;
   const bool fp8 = (d->flags & KVSHOT_TARGET_FP8) != 0;
-  const bool tmaps = fp8 ? encode_rows_fp8(&maps.tk, target_k, trows, tbox) &&
-                               encode_rows_fp8(&maps.tv, target_v, trows, tbox)
-                         : encode_rows(&maps.tk, target_k, trows, tbox) && encode_rows(&maps.tv, target_v, trows, tbox);
-  if (!tmaps || !encode_rows(&maps.dk, draft_k, drows, kDraftBoxRows) ||
-      !encode_rows(&maps.dv, draft_v, drows, kDraftBoxRows))
-    return KVSHOT_ERR_CUDA;
-  if (pl.kernel == Kernel::kTensorMemory) {
+  // The tensor-memory kernel stages tiles in the grouped layout: target tiles whenever their rows
+  // start on a multiple of 8 (always when paged; contiguous caches with l_cap % 8 == 0), draft tiles always.
+  const bool tmem_kernel = pl.kernel == Kernel::kTensorMemory;
+  const bool prefix_grouped = tmem_kernel && (paged || d->l_cap % 8 == 0);
+  bool tmaps;
+  if (fp8) {
+    tmaps = encode_rows_fp8(&maps.tk, target_k, trows, tbox) && encode_rows_fp8(&maps.tv, target_v, trows, tbox);
+  } else if (prefix_grouped) {
+    const uint32_t groups = (paged ? std::min(d->page_size, kTileKeys) : kTileKeys) / 8;
+    tmaps = encode_rows_grouped(&maps.tk, target_k, trows, groups) &&
+            encode_rows_grouped(&maps.tv, target_v, trows, groups);
+  } else {
+    tmaps = encode_rows(&maps.tk, target_k, trows, tbox) && encode_rows(&maps.tv, target_v, trows, tbox);
+  }
+  const bool dmaps = tmem_kernel ? encode_rows_group3(&maps.dk, draft_k, drows) &&
+                                       encode_rows_group3(&maps.dv, draft_v, drows)
+                                 : encode_rows(&maps.dk, draft_k, drows, kDraftBoxRows) &&
+                                       encode_rows(&maps.dv, draft_v, drows, kDraftBoxRows);
+  if (!tmaps || !dmaps) return KVSHOT_ERR_CUDA;
+  if (tmem_kernel) {
     if (!encode_q(&maps.q, q, d->num_caches, d->n_query, d->hq, q_box(d->hq / d->hkv, pl.nq_box, pl.spread)))
       return KVSHOT_ERR_CUDA;
   } else {
@@ -344,6 +402,7 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   p.qscale = static_cast<float>(scale * 1.4426950408889634);
   p.num_ctas = pl.num_ctas;
   p.fp8 = fp8 ? 1 : 0;
+  p.prefix_grouped = prefix_grouped ? 1 : 0;
   p.k_scale = fp8 ? std::ldexp(1.f, d->k_scale_exp) : 1.f;
   p.v_scale = fp8 ? std::ldexp(1.f, d->v_scale_exp) : 1.f;
 

@@ -33,6 +33,13 @@ constexpr int kDraftBoxRows = 8;                      // draft K/V are loaded 8 
 constexpr int kCcRows = 4;                            // rows per unit of the CUDA-core kernel
 constexpr int kMmaMaxTiles = 4;                       // m16 tiles per unit of the tensor-core kernel
 constexpr int kSpreadMaxRows = 64;                    // tensor-memory kernel: units up to this many rows are spread
+// Grouped tile layout of the tensor-memory kernel: a K (or V) tile is 8 groups
+// of 8 keys; group g starts at byte g * kGroupBytes and holds its keys' dims
+// 0..63 (1 KB, 128-byte swizzled rows) then dims 64..127 (kGroupHalfBytes on).
+// One TMA box then brings whole groups with both halves, e.g. a whole
+// 16-token page in one 4 KB box.
+constexpr int kGroupBytes = 8 * 256;
+constexpr int kGroupHalfBytes = 8 * 128;
 
 // Query box of the tensor-memory kernel's 4-D q map {128, hq, Nq, C}: `heads`
 // heads of the KV group x `nodes` draft nodes.  Dense units load all G x nq_box
@@ -70,6 +77,7 @@ struct AttnParams {
   float qscale;             // softmax scale * log2(e): scores are kept in the log2 domain
   int num_ctas;             // persistent grid size
   int fp8;                  // target K/V are e4m3 codes (KVSHOT_TARGET_FP8; m16n8k16 kernel only)
+  int prefix_grouped;       // tensor-memory kernel: prefix tiles are staged in the grouped layout (draft tiles always)
   float k_scale, v_scale;   // fp8: 2^k_scale_exp, 2^v_scale_exp
 };
 
@@ -89,6 +97,10 @@ struct AppendParams {
   float eps;
 };
 
+// Target and draft K/V maps.  The m16n8k16 and CUDA-core kernels use 2-D
+// maps (boxes of one 64-dim half); the tensor-memory kernel uses grouped maps
+// (4-D target, 3-D draft: boxes of whole 8-key groups, both halves) except
+// for a contiguous target cache whose l_cap is not a multiple of 8.
 struct TensorMaps {
   CUtensorMap tk, tv, dk, dv;
   CUtensorMap q;  // [C, Nq, hq, 128] as 4-D {128, hq, Nq, C}; used by the tensor-memory kernel
