@@ -109,6 +109,12 @@ typedef struct kvshot_attn_desc {
   int32_t* err_flag;         /* optional device int32, 0 before the call; see conventions above */
   int32_t k_scale_exp;       /* KVSHOT_TARGET_FP8: target keys are e4m3 x 2^k_scale_exp, |exp| <= 64 */
   int32_t v_scale_exp;       /* KVSHOT_TARGET_FP8: target values are e4m3 x 2^v_scale_exp, |exp| <= 64 */
+  uint32_t wait_limit_ns;    /* watchdog: longest any one wait of the attention kernels' load/compute
+                                pipeline may take, in ns; 0 = 2 s.  A wait that runs past it records
+                                KVSHOT_ERR_TIMEOUT; the kernel then stops computing, waits (2 s at most
+                                each) for the copies and tensor-core operations it already issued, and
+                                returns, leaving the outputs unspecified.  Setting it near zero makes every
+                                CTA give up on its first unfinished wait: a way to exercise that path. */
 } kvshot_attn_desc;
 
 /*
@@ -169,7 +175,11 @@ kvshot_status kvshot_draft_attn(const kvshot_attn_desc* desc, const void* q, con
  *    (kvshot_draft_attn_workspace_size(desc) > KVSHOT_STATIC_WORKSPACE_BYTES)
  *    are rejected with KVSHOT_ERR_WORKSPACE before anything is launched.
  *  - The first call on each device looks up the array's device address (with
- *    that device current); make that first call before any stream capture.
+ *    that device current) and keeps it for the life of the process; make that
+ *    first call before any stream capture.  The kept address belongs to the
+ *    device's primary context: after cudaDeviceReset (or any teardown of that
+ *    context) it is stale, and the entry point must not be called again in
+ *    that process.
  *  - All calls on a device share the one array and it keeps the last call's
  *    contents.  Nothing in it has to start at zero, but two calls whose
  *    kernels overlap on the GPU (e.g. on different streams without ordering)
@@ -182,9 +192,10 @@ kvshot_status kvshot_draft_attn_static(const kvshot_attn_desc* desc, const void*
 
 /*
  * Draft append with RoPE: the drafter's new K/V for draft positions j > t
- * enter M_i (App. B: "the drafter generates its own KV via learned
- * projections"; the projections themselves are upstream GEMMs), with rotary
- * position embedding applied to q and k (RoPE re-application, Sec. 3.2).
+ * enter M_i (App. B: past the verified prefix the memory holds keys and
+ * values that the drafter computes itself with its own projection weights;
+ * those projections are upstream GEMMs), with rotary position embedding
+ * applied to q and k (RoPE re-application, Sec. 3.2).
  *
  * For cache c and new node i in [0, n_new) at position pos = positions[c, i]:
  *   theta_j = pos * rope_base^(-2j / 128),  j in [0, 64)

@@ -204,10 +204,11 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
     // After a timed-out wait the warp keeps walking the tiles (so every named
     // barrier is still met) but waits for and computes nothing more.
     bool live = !*pipe.abort;
-    if (live && !mbar_wait(smem_addr(&pipe.full[stage]), phase, p.err)) {
+    if (live && !mbar_wait(smem_addr(&pipe.full[stage]), phase, p.err, p.wait_ns)) {
       *pipe.abort = 1;
       live = false;
     }
+    live = __all_sync(0xffffffffu, live);  // the warp-wide MMA and shuffle steps below need the whole warp
     const uint32_t kbase = smem_addr(pipe.ring + static_cast<size_t>(stage) * kStageBytes);
     const uint32_t vbase = kbase + kKVTileBytes;
     const int kw0 = warp * kKeysPerWarp;

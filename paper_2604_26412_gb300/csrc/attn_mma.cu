@@ -329,10 +329,11 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
       }
     }
     bool live = !*pipe.abort;
-    if (live && !mbar_wait(smem_addr(&pipe.full[stage]), phase, p.err)) {
+    if (live && !mbar_wait(smem_addr(&pipe.full[stage]), phase, p.err, p.wait_ns)) {
       *pipe.abort = 1;
       live = false;
     }
+    live = __all_sync(0xffffffffu, live);  // the warp-wide MMA and shuffle steps below need the whole warp
     uint8_t* kptr = pipe.ring + static_cast<size_t>(stage) * kStageBytes;
     const uint32_t kbase = smem_addr(kptr);
     const uint32_t vbase = kbase + kKVTileBytes;

@@ -149,9 +149,9 @@ __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, 
   for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
     bool ok = !*pipe.abort;
-    if (ok && ti.first) ok = mbar_wait(smem_addr(sm.qfull), piece & 1, p.err);
-    if (ok && t >= kNS) ok = mbar_wait(smem_addr(&sm.sfree[t % kNS]), ((t - kNS) / kNS) & 1, p.err);
-    if (ok) ok = mbar_wait(smem_addr(&sm.kfull[t % kNK]), (t / kNK) & 1, p.err);
+    if (ok && ti.first) ok = mbar_wait(smem_addr(sm.qfull), piece & 1, p.err, p.wait_ns);
+    if (ok && t >= kNS) ok = mbar_wait(smem_addr(&sm.sfree[t % kNS]), ((t - kNS) / kNS) & 1, p.err, p.wait_ns);
+    if (ok) ok = mbar_wait(smem_addr(&sm.kfull[t % kNK]), (t / kNK) & 1, p.err, p.wait_ns);
     if (!ok) {
       *pipe.abort = 1;
       break;
@@ -192,9 +192,9 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
     }
     const bool first = t - piece_t0 < 2;
     bool ok = !*pipe.abort;
-    if (ok && first && piece > 1) ok = mbar_wait(smem_addr(sm.ofree), (piece - 2) & 1, p.err);
-    if (ok) ok = mbar_wait(smem_addr(&sm.pfull[t % kNP]), (t / kNP) & 1, p.err);
-    if (ok) ok = mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err);
+    if (ok && first && piece > 1) ok = mbar_wait(smem_addr(sm.ofree), (piece - 2) & 1, p.err, p.wait_ns);
+    if (ok) ok = mbar_wait(smem_addr(&sm.pfull[t % kNP]), (t / kNP) & 1, p.err, p.wait_ns);
+    if (ok) ok = mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err, p.wait_ns);
     if (!ok) {
       *pipe.abort = 1;
       break;
@@ -236,7 +236,7 @@ template <bool kSpread>
 __device__ __forceinline__ void rescale_o_tmem(const Smem& sm, const Pipe& pipe, const AttnParams& p, uint32_t my_o,
                                                int t, float alpha) {
   constexpr int kOChunks = kSpread ? 2 : 4;  // 32-column O chunks per thread
-  if (!mbar_wait(smem_addr(&sm.pvdone[(t - 2) % kNP]), ((t - 2) / kNP) & 1, p.err)) *pipe.abort = 1;
+  if (!mbar_wait(smem_addr(&sm.pvdone[(t - 2) % kNP]), ((t - 2) / kNP) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
   tc_fence_after();
 #pragma unroll
   for (int c = 0; c < kOChunks; ++c) {
@@ -309,7 +309,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
     bool live = !*pipe.abort;
     if ((t & 1) == wg) {
       const int sbuf = t % kNS, b = t % kNP;
-      if (live && !mbar_wait(smem_addr(&sm.sfull[sbuf]), (t / kNS) & 1, p.err)) {
+      if (live && !mbar_wait(smem_addr(&sm.sfull[sbuf]), (t / kNS) & 1, p.err, p.wait_ns)) {
         *pipe.abort = 1;
         live = false;
       }
@@ -392,7 +392,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
       }
       // The P buffer is free once P.V of tile t - kNP has completed.
-      if (live && t >= kNP && !mbar_wait(smem_addr(&sm.pvdone[b]), ((t - kNP) / kNP) & 1, p.err)) *pipe.abort = 1;
+      if (live && t >= kNP && !mbar_wait(smem_addr(&sm.pvdone[b]), ((t - kNP) / kNP) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
       if (live && valid) {
         uint8_t* prow = sm.pbuf + b * kPBufBytes + tl * 128;
 #pragma unroll
@@ -411,7 +411,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       }
       if (live && ti.nkeys < kTileKeys) {
         // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.
-        if (!mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err)) *pipe.abort = 1;
+        if (!mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
         uint8_t* vptr = sm.vring + static_cast<size_t>(t % kNV) * kKVBytes;
         const int nz = (kTileKeys - ti.nkeys) * 16;
         for (int i = wtid; i < nz; i += kSoftmaxThreads / 2) {
@@ -430,8 +430,8 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       // from tile t - 6's by parity, so it first waits P.V of its own tile t - 1.
       bool ok = live;
       if (ok && (t & 1) != wg && t >= 1)
-        ok = mbar_wait(smem_addr(&sm.pvdone[(t - 1) % kNP]), ((t - 1) / kNP) & 1, p.err);
-      ok = ok && mbar_wait(smem_addr(&sm.pvdone[t % kNP]), (t / kNP) & 1, p.err);
+        ok = mbar_wait(smem_addr(&sm.pvdone[(t - 1) % kNP]), ((t - 1) / kNP) & 1, p.err, p.wait_ns);
+      ok = ok && mbar_wait(smem_addr(&sm.pvdone[t % kNP]), (t / kNP) & 1, p.err, p.wait_ns);
       ok = __all_sync(0xffffffffu, ok);
       tc_fence_after();
       float l_row = l_run;
@@ -634,7 +634,7 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
       }
       if (lane == 0) {
         const uint32_t qbar = smem_addr(sm.qfull);
-        ok = mbar_wait(smem_addr(sm.qempty), (piece & 1) ^ 1u, p.err) && !*pipe.abort;
+        ok = mbar_wait(smem_addr(sm.qempty), (piece & 1) ^ 1u, p.err, p.wait_ns) && !*pipe.abort;
         if (ok) {
           const int rb = cu.hr - h * p.row_blocks;
           const uint32_t dst = smem_addr(sm.qbuf);
@@ -673,7 +673,7 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
       const bool need = lane == 1 || t >= kNK;
       const uint32_t bar = lane == 0 ? smem_addr(&sm.sfull[(t - kNK) % kNS]) : smem_addr(&sm.vempty[vslot]);
       const uint32_t par = lane == 0 ? (((t - kNK) / kNS) & 1) : (((t / kNV) & 1) ^ 1u);
-      ok = (!need || mbar_wait(bar, par, p.err)) && !*pipe.abort;
+      ok = (!need || mbar_wait(bar, par, p.err, p.wait_ns)) && !*pipe.abort;
     }
     ok = __all_sync(0xffffffffu, ok);
     if (!ok) {
@@ -767,8 +767,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
       if (stream == 0) run_mma_qk(p, sm, pipe, tmem, cu);
       else run_mma_pv(p, sm, pipe, tmem, cu);
-      // Every MMA must have completed before TMEM is released.
-      mbar_wait(smem_addr(&sm.mmadone[stream]), 0, p.err);
+      // Every MMA must have completed before TMEM is released.  Each MMA issued reads shared memory
+      // whose loads it already waited for, so it finishes; the wait is retried (bounded) if it runs
+      // past its limit rather than freeing TMEM under a running MMA.
+      for (int k = 0; k < 4 && !mbar_wait(smem_addr(&sm.mmadone[stream]), 0, p.err); ++k) {
+      }
     }
     __syncwarp();
   } else if (warp < 8) {

@@ -403,6 +403,7 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   p.num_ctas = pl.num_ctas;
   p.fp8 = fp8 ? 1 : 0;
   p.prefix_grouped = prefix_grouped ? 1 : 0;
+  p.wait_ns = d->wait_limit_ns != 0 ? d->wait_limit_ns : static_cast<uint32_t>(2000000000u);
   p.k_scale = fp8 ? std::ldexp(1.f, d->k_scale_exp) : 1.f;
   p.v_scale = fp8 ? std::ldexp(1.f, d->v_scale_exp) : 1.f;
 

@@ -59,25 +59,24 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return done != 0;
 }
 
-// Every pipeline wait gives up after this long, records KVSHOT_ERR_TIMEOUT
-// and lets the kernel wind down instead of spinning forever.
+// Every wait gives up after a time limit, records KVSHOT_ERR_TIMEOUT and lets
+// the kernel wind down instead of spinning forever.  The attention kernels'
+// pipeline waits take the call's limit (AttnParams::wait_ns); waits for work
+// already issued (the drain of in-flight copies after an abort, the last
+// tensor-core operations before TMEM is freed) and the other kernels' waits
+// take kWaitLimitNs.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
-__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int32_t* err) {
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int32_t* err, uint64_t limit_ns) {
   const uint64_t t0 = global_timer_ns();
   for (;;) {
     for (int i = 0; i < 64; ++i)
       if (mbar_try_wait(bar, parity)) return true;
-    if (global_timer_ns() - t0 > kWaitLimitNs) {
+    if (global_timer_ns() - t0 > limit_ns) {
       set_error(err, KVSHOT_ERR_TIMEOUT);
       return false;
     }
   }
-}
-
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t* err) {
-  if (mbar_try_wait(bar, parity)) return true;
-  return mbar_wait_slow(bar, parity, err);
 }
 
 // Non-blocking test of a phase's completion.
@@ -91,6 +90,29 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
       : "r"(bar), "r"(parity)
       : "memory");
   return done != 0;
+}
+
+// Limits below this are polled with the non-blocking test and a timer check
+// on every iteration (mbarrier.try_wait may suspend the thread for longer than
+// such a limit, so the timer would never be looked at in time).
+constexpr uint64_t kPollBelowNs = 100000;
+
+__device__ __noinline__ bool mbar_wait_poll(uint32_t bar, uint32_t parity, int32_t* err, uint64_t limit_ns) {
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    if (mbar_test_wait(bar, parity)) return true;
+    if (global_timer_ns() - t0 > limit_ns) {
+      set_error(err, KVSHOT_ERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t* err,
+                                          uint64_t limit_ns = kWaitLimitNs) {
+  if (limit_ns < kPollBelowNs) return mbar_wait_poll(bar, parity, err, limit_ns);
+  if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, err, limit_ns);
 }
 
 // Programmatic dependent launch.  The attention kernels let the kernel that
@@ -479,7 +501,7 @@ __device__ __forceinline__ void run_producer(const AttnParams& p, const TensorMa
       if (lane == 0) {
         const int qb = piece % qp->nbuf;
         const uint32_t qbar = smem_addr(&qp->full[qb]);
-        ok = mbar_wait(smem_addr(&qp->empty[qb]), ((piece / qp->nbuf) & 1) ^ 1u, p.err) ? 1 : 0;
+        ok = mbar_wait(smem_addr(&qp->empty[qb]), ((piece / qp->nbuf) & 1) ^ 1u, p.err, p.wait_ns) ? 1 : 0;
         if (ok && !*pipe.abort) {
           const int rb = cu.hr - h * p.row_blocks;
           const uint32_t dst = smem_addr(qp->buf + qb * kQBufBytes);
@@ -494,7 +516,7 @@ __device__ __forceinline__ void run_producer(const AttnParams& p, const TensorMa
       ++piece;
     }
     if (lane == 0 && ok) {
-      ok = mbar_wait(smem_addr(&pipe.empty[stage]), phase ^ 1u, p.err) ? 1 : 0;
+      ok = mbar_wait(smem_addr(&pipe.empty[stage]), phase ^ 1u, p.err, p.wait_ns) ? 1 : 0;
       if (!ok || *pipe.abort) ok = 0;
     }
     ok = __shfl_sync(0xffffffffu, ok, 0);

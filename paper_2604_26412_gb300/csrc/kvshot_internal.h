@@ -78,6 +78,7 @@ struct AttnParams {
   int num_ctas;             // persistent grid size
   int fp8;                  // target K/V are e4m3 codes (KVSHOT_TARGET_FP8; m16n8k16 kernel only)
   int prefix_grouped;       // tensor-memory kernel: prefix tiles are staged in the grouped layout (draft tiles always)
+  uint32_t wait_ns;         // limit on any one pipeline wait (desc->wait_limit_ns, default 2 s)
   float k_scale, v_scale;   // fp8: 2^k_scale_exp, 2^v_scale_exp
 };
 

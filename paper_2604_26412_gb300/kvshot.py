@@ -72,6 +72,7 @@ class AttnDesc(ctypes.Structure):
         ("err_flag", ctypes.c_void_p),
         ("k_scale_exp", ctypes.c_int32),
         ("v_scale_exp", ctypes.c_int32),
+        ("wait_limit_ns", ctypes.c_uint32),
     ]
 
 
@@ -187,11 +188,12 @@ def _stream(stream) -> Optional[int]:
 
 def make_desc(*, num_caches, num_seqs, hq, hkv, n_nodes, n_query, n_max, max_seq_len, head_dim=128, page_size=0,
               max_pages_per_seq=0, num_pages=0, l_cap=0, scale=0.0, tree=False, flags=0, num_ctas=0,
-              workspace=None, workspace_bytes=0, err_flag=None, k_scale_exp=0, v_scale_exp=0) -> AttnDesc:
+              workspace=None, workspace_bytes=0, err_flag=None, k_scale_exp=0, v_scale_exp=0,
+              wait_limit_ns=0) -> AttnDesc:
     f = int(flags) | (KVSHOT_TREE if tree else 0)
     return AttnDesc(num_caches, num_seqs, hq, hkv, head_dim, page_size, max_pages_per_seq, num_pages, l_cap,
                     max_seq_len, n_nodes, n_query, n_max, float(scale), f, num_ctas, _ptr(workspace),
-                    int(workspace_bytes), _ptr(err_flag), int(k_scale_exp), int(v_scale_exp))
+                    int(workspace_bytes), _ptr(err_flag), int(k_scale_exp), int(v_scale_exp), int(wait_limit_ns))
 
 
 def workspace_size(desc: AttnDesc) -> int:
