@@ -54,6 +54,18 @@ constexpr uint32_t kTmemO = kNS * kTileKeys;
 constexpr int kMiscInts = 12;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max grows by > 256x
 
+// Row modes.  Dense: one block of up to 128 stacked rows, one thread per TMEM lane, the two
+// warpgroups alternating tiles.  Spread: up to 64 rows, 16 per TMEM lane quarter.  Pair: two
+// 128-row blocks of one KV head (129..256 rows), warpgroup w owning block w on every tile.
+constexpr int kModeDense = 0, kModeSpread = 1, kModePair = 2;
+constexpr int kPairNK = 4;                 // paired blocks: K tiles in flight
+constexpr int kPairNV = 5;                 // paired blocks: V tiles in flight
+template <int M>
+struct RingOf {
+  static constexpr int NK = M == kModePair ? kPairNK : kNK;
+  static constexpr int NV = M == kModePair ? kPairNV : kNV;
+};
+
 // Byte offset of 16-byte chunk `ch` (dims 8ch..8ch+7) of key r in a K or V
 // tile of either layout (128-byte swizzle: chunk index XOR row index mod 8).
 __device__ __forceinline__ uint32_t tile_off_tc(int r, int ch, bool grouped) {
@@ -601,9 +613,11 @@ __device__ __forceinline__ TileBoxes tile_boxes(const AttnParams& p, const Curso
 // boxes of 16 stacked rows, box k to TMEM lanes (= q buffer rows)
 // 32 k .. 32 k + 15.  misc[8 + role] / misc[10 + role]: one past the last K /
 // V tile this warp issued (read by the drain after an abort).
-template <bool kSpread>
-__device__ __forceinline__ void run_producer_tc(const AttnParams& p, const TensorMaps& maps, const Smem& sm,
+template <int kMode, class SM>
+__device__ __forceinline__ void run_producer_tc(const AttnParams& p, const TensorMaps& maps, const SM& sm,
                                                 const Pipe& pipe, Cursor cu, int nq_box, int role) {
+  constexpr bool kSpread = kMode == kModeSpread;
+  constexpr int NK = RingOf<kMode>::NK, NV = RingOf<kMode>::NV;
   const int lane = threadIdx.x & 31;
   const uint64_t policy = l2_policy_evict_first();
   PageWindow win;
@@ -638,15 +652,26 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
         if (ok) {
           const int rb = cu.hr - h * p.row_blocks;
           const uint32_t dst = smem_addr(sm.qbuf);
-          const QBox qb = q_box(p.G, nq_box, kSpread);
-          const int box_rows = qb.heads * qb.nodes;
-          const int nqb = kSpread ? (rows_q + box_rows - 1) / box_rows : 1;
-          mbar_arrive_expect_tx(qbar, 2 * nqb * box_rows * 128);
-          for (int k = 0; k < nqb; ++k) {
-            const int s0 = k * box_rows;  // first stacked row of the box
-            const uint32_t d = dst + k * 32 * 128;
-            tma_load_4d(d, &maps.q, 0, h * p.G + s0 % p.G, rb * nq_box + s0 / p.G, cu.c, qbar);
-            tma_load_4d(d + kQRows * 128, &maps.q, 64, h * p.G + s0 % p.G, rb * nq_box + s0 / p.G, cu.c, qbar);
+          if constexpr (kMode == kModePair) {
+            // Q_0 and Q_1: the unit's two blocks of nq_box draft nodes x G heads (128 rows each).
+            mbar_arrive_expect_tx(qbar, 4 * kQRows * 128);
+            for (int w = 0; w < 2; ++w) {
+              const uint32_t d = dst + w * kQBufBytes;
+              const int node0 = (2 * rb + w) * nq_box;
+              tma_load_4d(d, &maps.q, 0, h * p.G, node0, cu.c, qbar);
+              tma_load_4d(d + kQRows * 128, &maps.q, 64, h * p.G, node0, cu.c, qbar);
+            }
+          } else {
+            const QBox qb = q_box(p.G, nq_box, kSpread);
+            const int box_rows = qb.heads * qb.nodes;
+            const int nqb = kSpread ? (rows_q + box_rows - 1) / box_rows : 1;
+            mbar_arrive_expect_tx(qbar, 2 * nqb * box_rows * 128);
+            for (int k = 0; k < nqb; ++k) {
+              const int s0 = k * box_rows;  // first stacked row of the box
+              const uint32_t d = dst + k * 32 * 128;
+              tma_load_4d(d, &maps.q, 0, h * p.G + s0 % p.G, rb * nq_box + s0 / p.G, cu.c, qbar);
+              tma_load_4d(d + kQRows * 128, &maps.q, 64, h * p.G + s0 % p.G, rb * nq_box + s0 / p.G, cu.c, qbar);
+            }
           }
           sm.misc[3] = piece + 1;
         }
@@ -666,13 +691,26 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
     }
     // Lanes 0..15 load the K boxes, lanes 16..31 the V boxes (box = lane & 15).
     const int kv = lane >> 4, i = lane & 15;
-    const int kslot = t % kNK, vslot = t % kNV;
+    const int kslot = t % NK, vslot = t % NV;
     // A V slot is free once P.V of its previous tile completed, a K slot once QK^T of its previous tile
-    // (t - kNK) completed.  Lane 0 waits for the K slot and lane 1 for the V slot together.
+    // (t - NK) completed.  Lane 0 waits for the K slot and lane 1 for the V slot together.  Single
+    // blocks read the K-slot release off the S buffer of tile t - NK, whose next completion (tile t)
+    // needs this very K tile, so its phase cannot be mistaken for one two phases later.  Paired blocks
+    // have only two S buffers per block (tile t - NK + 2 < t may complete first), so their K slots
+    // have release barriers of their own.
     if (lane < 2 && ok) {
-      const bool need = lane == 1 || t >= kNK;
-      const uint32_t bar = lane == 0 ? smem_addr(&sm.sfull[(t - kNK) % kNS]) : smem_addr(&sm.vempty[vslot]);
-      const uint32_t par = lane == 0 ? (((t - kNK) / kNS) & 1) : (((t / kNV) & 1) ^ 1u);
+      const bool need = lane == 1 || t >= NK || kMode == kModePair;
+      const int tk = t - NK;
+      uint32_t kbar, kpar;
+      if constexpr (kMode == kModePair) {
+        kbar = smem_addr(&sm.kempty[kslot]);
+        kpar = ((t / NK) & 1) ^ 1u;
+      } else {
+        kbar = smem_addr(&sm.sfull[tk % kNS]);
+        kpar = (tk / kNS) & 1;
+      }
+      const uint32_t bar = lane == 0 ? kbar : smem_addr(&sm.vempty[vslot]);
+      const uint32_t par = lane == 0 ? kpar : (((t / NV) & 1) ^ 1u);
       ok = (!need || mbar_wait(bar, par, p.err, p.wait_ns)) && !*pipe.abort;
     }
     ok = __all_sync(0xffffffffu, ok);
@@ -699,6 +737,453 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
       break;
     }
   }
+}
+
+
+// ============================================================ paired row blocks
+//
+// Stacks of 129..256 rows per KV head (whole-tree and whole-chain query modes):
+// a unit holds two 128-row blocks of one KV head, so each K/V tile leaves HBM
+// once for both.  Warpgroup w owns block w on every tile: S_w = Q_w K^T into
+// its own two S buffers, its own online softmax, O_w += P_w V into its own
+// accumulator and its own epilogue (no merge between the warpgroups).
+// TMEM: S_{w,j} (tile parity j) at columns 64 (2 w + j), O_w at 256 + 128 w.
+// P stays in tensor memory: the softmax writes P_w (bf16 pairs, 32 columns)
+// over the S columns it has read, and P.V takes its A operand from there, so
+// the softmax of the next tile never waits for this tile's P.V, and S buffer
+// (w, j) is released when P.V of its tile completes.
+
+struct SmemPair {
+  uint8_t* kring;      // kPairNK x K tile
+  uint8_t* vring;      // kPairNV x V tile
+  uint8_t* qbuf;       // Q_0, Q_1 (kQBufBytes each)
+  uint64_t* kfull;     // [kPairNK]  TMA -> QK^T issuer
+  uint64_t* kempty;    // [kPairNK]  both QK^T of the tile completed -> TMA
+  uint64_t* vfull;     // [kPairNV]  TMA -> P.V issuer (and warpgroup 0 on partial tiles)
+  uint64_t* vempty;    // [kPairNV]  both P.V of the tile completed -> TMA
+  uint64_t* qfull;     // [1]
+  uint64_t* qempty;    // [1]
+  uint64_t* sfull;     // [4]  S_{w,j} written (index 2 w + j)
+  uint64_t* sfree;     // [4]  P.V of the tile in S_{w,j} completed: the buffer is free
+  uint64_t* pfull;     // [4]  P_w of a tile with parity j written over S_{w,j} (128 threads)
+  uint64_t* pvdone;    // [2]  O_w += P_w V completed
+  uint64_t* ofree;     // [2]  warpgroup w's epilogue read O_w (128 threads)
+  uint64_t* mmadone;   // [2]
+  uint64_t* anc;       // [64]
+  int* par;            // [64]
+  uint32_t* tmem_base;
+  int* misc;           // as Smem::misc
+  int* len;
+  int* base;
+};
+
+__host__ __device__ inline size_t smem_bytes_pair(int C) {
+  size_t off = static_cast<size_t>(kPairNK + kPairNV) * kKVBytes + 2 * kQBufBytes;
+  off += sizeof(uint64_t) * (2 * kPairNK + 2 * kPairNV + 2 + 4 + 4 + 4 + 2 + 2 + 2);
+  off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
+  off += sizeof(uint32_t) * 4 + sizeof(int) * kMiscInts;
+  off += sizeof(int) * (2 * C + 1);
+  return off + 1024;
+}
+
+__device__ SmemPair carve_pair(uint8_t* raw, int C) {
+  SmemPair s;
+  uint8_t* p = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
+  s.kring = p;
+  p += kPairNK * kKVBytes;
+  s.vring = p;
+  p += kPairNV * kKVBytes;
+  s.qbuf = p;
+  p += 2 * kQBufBytes;
+  uint64_t* b = reinterpret_cast<uint64_t*>(p);
+  s.kfull = b;
+  s.kempty = s.kfull + kPairNK;
+  s.vfull = s.kempty + kPairNK;
+  s.vempty = s.vfull + kPairNV;
+  s.qfull = s.vempty + kPairNV;
+  s.qempty = s.qfull + 1;
+  s.sfull = s.qempty + 1;
+  s.sfree = s.sfull + 4;
+  s.pfull = s.sfree + 4;
+  s.pvdone = s.pfull + 4;
+  s.ofree = s.pvdone + 2;
+  s.mmadone = s.ofree + 2;
+  s.anc = s.mmadone + 2;
+  s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
+  s.tmem_base = reinterpret_cast<uint32_t*>(s.par + kMaxTreeNodes);
+  s.misc = reinterpret_cast<int*>(s.tmem_base + 4);
+  s.len = s.misc + kMiscInts;
+  s.base = s.len + C;
+  return s;
+}
+
+// S_w = Q_w K^T of every tile for w = 0, 1.  Tile t needs its K tile, the
+// piece's q blocks (first tile of a piece) and, per block, S buffer (w, t & 1)
+// freed by the completion of P.V of tile t - 2.
+__device__ __forceinline__ void run_mma_qk_pair(const AttnParams& p, const SmemPair& sm, const Pipe& pipe,
+                                                uint32_t tmem, Cursor cu) {
+  constexpr uint32_t idesc = idesc_bf16(128, 64, false);
+  int piece = 0;
+  for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
+    const TileInfo ti = tile_info(cu, p);
+    const int j = t & 1;
+    bool ok = !*pipe.abort;
+    if (ok && ti.first) ok = mbar_wait(smem_addr(sm.qfull), piece & 1, p.err, p.wait_ns);
+    if (ok) ok = mbar_wait(smem_addr(&sm.kfull[t % kPairNK]), (t / kPairNK) & 1, p.err, p.wait_ns);
+    if (!ok) {
+      *pipe.abort = 1;
+      break;
+    }
+    if (ti.first) sm.misc[4] = ++piece;
+    sm.misc[2] = t + 1;
+    const uint32_t kbase = smem_addr(sm.kring + static_cast<size_t>(t % kPairNK) * kKVBytes);
+    const bool grouped = ti.draft || p.prefix_grouped;
+    const uint32_t half_off = grouped ? kGroupHalfBytes : kHalfBytes, group_off = grouped ? kGroupBytes : 1024;
+    for (int w = 0; w < 2; ++w) {
+      if (t >= 2 && !mbar_wait(smem_addr(&sm.sfree[2 * w + j]), ((t - 2) >> 1) & 1, p.err, p.wait_ns)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t qbase = smem_addr(sm.qbuf + w * kQBufBytes);
+#pragma unroll
+      for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+        const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
+        const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * half_off + (ks & 3) * 32, 16, group_off);
+        tc_mma(tmem + (2 * w + j) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
+      }
+      tc_commit(smem_addr(&sm.sfull[2 * w + j]));
+    }
+    if (!ok) {
+      *pipe.abort = 1;
+      break;
+    }
+    tc_commit(smem_addr(&sm.kempty[t % kPairNK]));
+    if (ti.last) tc_commit(smem_addr(sm.qempty));
+  }
+  tc_commit(smem_addr(&sm.mmadone[0]));
+}
+
+// O_w += P_w V of every tile for w = 0, 1, with P_w read from tensor memory
+// (the S columns of the tile).  The first P.V into O_w of a piece (which
+// overwrites O_w) needs the previous piece's epilogue to have read O_w.  Each
+// completion frees S buffer (w, t & 1) for QK^T of tile t + 2.
+__device__ __forceinline__ void run_mma_pv_pair(const AttnParams& p, const SmemPair& sm, const Pipe& pipe,
+                                                uint32_t tmem, Cursor cu) {
+  constexpr uint32_t idesc = idesc_bf16(128, 128, true);
+  int piece = 0, piece_t0 = 0;
+  for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
+    const TileInfo ti = tile_info(cu, p);
+    const int j = t & 1;
+    if (ti.first) {
+      ++piece;
+      piece_t0 = t;
+    }
+    bool ok = !*pipe.abort;
+    if (ok) ok = mbar_wait(smem_addr(&sm.vfull[t % kPairNV]), (t / kPairNV) & 1, p.err, p.wait_ns);
+    if (!ok) {
+      *pipe.abort = 1;
+      break;
+    }
+    sm.misc[6] = t + 1;
+    const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(t % kPairNV) * kKVBytes);
+    const bool grouped = ti.draft || p.prefix_grouped;
+    const uint32_t half_off = grouped ? kGroupHalfBytes : kHalfBytes, group_off = grouped ? kGroupBytes : 1024;
+    for (int w = 0; w < 2; ++w) {
+      if (t == piece_t0 && piece > 1) ok = mbar_wait(smem_addr(&sm.ofree[w]), (piece - 2) & 1, p.err, p.wait_ns);
+      if (ok) ok = mbar_wait(smem_addr(&sm.pfull[2 * w + j]), (t >> 1) & 1, p.err, p.wait_ns);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t pcol = tmem + (2 * w + j) * kTileKeys;  // P_w: 32 columns of bf16 pairs
+      const uint32_t o = tmem + kTmemO + 128 * w;
+#pragma unroll
+      for (int k16 = 0; k16 < kTileKeys / 16; ++k16) {
+        const uint64_t bd = smem_desc_sw128(vbase + k16 * 2 * group_off, half_off, group_off);
+        tc_mma_tmem_a(o, pcol + 8 * k16, bd, idesc, (t == piece_t0 && k16 == 0) ? 0u : 1u);
+      }
+      tc_commit(smem_addr(&sm.pvdone[w]));
+      tc_commit(smem_addr(&sm.sfree[2 * w + j]));
+    }
+    if (!ok) {
+      *pipe.abort = 1;
+      break;
+    }
+    tc_commit(smem_addr(&sm.vempty[t % kPairNV]));
+  }
+  tc_commit(smem_addr(&sm.mmadone[1]));
+}
+
+// Softmax and epilogue of warpgroup wg = block wg of every unit: thread =
+// TMEM lane = row r of the block, all 64 S columns of a tile.
+__device__ __forceinline__ void run_softmax_pair(const AttnParams& p, const SmemPair& sm, const Pipe& pipe,
+                                                 uint32_t tmem, Cursor cu) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int quarter = warp & 3, wg = warp >> 2;
+  const int wtid = threadIdx.x & 127;
+  const int r = quarter * 32 + lane;
+  const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+  const uint32_t my_s = trow + 2 * wg * kTileKeys;  // S_{wg, j} at my_s + 64 j
+  const uint32_t my_o = trow + kTmemO + 128 * wg;
+  const int HR = p.hkv * p.row_blocks;
+  const float qscale = p.qscale;
+  const bool tree = p.tree != 0;
+  const int nq = p.Nq, n_nodes = p.N;
+  int unit_c = -1, unit_hr = -1, h = 0, rr = 0, nl = 0;
+  bool valid = false, warp_live = false;
+  float m_run = -INFINITY, l_run = 0.f;
+  int anc_seq = -1;
+  wait_for_prerequisite_grid();
+  for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
+    const TileInfo ti = tile_info(cu, p);
+    const int j = t & 1;
+    if (cu.c != unit_c || cu.hr != unit_hr) {
+      unit_c = cu.c;
+      unit_hr = cu.hr;
+      h = cu.hr / p.row_blocks;
+      const int rb = cu.hr - h * p.row_blocks;
+      const int row0 = rb * p.rows_per_unit + wg * kQRows;  // this warpgroup's first stacked row
+      rr = row0 + r;
+      valid = rr < p.rows_total;
+      warp_live = row0 + quarter * 32 < p.rows_total;
+      nl = valid ? rr / p.G : 0;
+    }
+    if (ti.first) {
+      m_run = -INFINITY;
+      l_run = 0.f;
+    }
+    if (ti.draft && tree) {
+      const int seq = cu.c / (p.C / p.B);
+      if (seq != anc_seq) {
+        build_ancestor_masks(p, seq, sm.anc, sm.par, threadIdx.x, kSoftmaxThreads, kBarSoftmax);
+        anc_seq = seq;
+      }
+    }
+    bool live = !*pipe.abort;
+    if (live && !mbar_wait(smem_addr(&sm.sfull[2 * wg + j]), (t >> 1) & 1, p.err, p.wait_ns)) {
+      *pipe.abort = 1;
+      live = false;
+    }
+    live = __all_sync(0xffffffffu, live);
+    tc_fence_after();
+    float pr[kTileKeys];
+    bool any_rescale = false;
+    float alpha = 1.f;
+    if (live && warp_live) {
+      uint32_t sv[kTileKeys];
+      tmem_ld32(my_s + j * kTileKeys, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+      tmem_ld32(my_s + j * kTileKeys + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+      tmem_wait_ld();
+      float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      if (valid && !ti.draft && ti.nkeys >= kTileKeys) {  // a full prefix tile: every key is visible
+#pragma unroll
+        for (int k = 0; k < kTileKeys; ++k) {
+          pr[k] = __uint_as_float(sv[k]) * qscale;
+          mx4[k & 3] = fmaxf(mx4[k & 3], pr[k]);
+        }
+      } else {
+        uint64_t vis = 0;
+        if (valid) {
+          vis = ti.nkeys >= 64 ? ~0ull : ((1ull << ti.nkeys) - 1ull);
+          if (ti.draft) {
+            uint64_t dm;
+            if (tree) {
+              dm = sm.anc[min(nl, nq - 1)] >> ti.key0;  // tree drafts have N <= 64, so key0 == 0
+            } else {
+              const int last = n_nodes - nq + nl - ti.key0;  // chain: slots key0 .. node are visible
+              dm = last >= 63 ? ~0ull : (last < 0 ? 0ull : ((2ull << last) - 1ull));
+            }
+            vis &= dm;
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < kTileKeys; ++k) {
+          pr[k] = ((vis >> k) & 1u) ? __uint_as_float(sv[k]) * qscale : -INFINITY;
+          mx4[k & 3] = fmaxf(mx4[k & 3], pr[k]);
+        }
+      }
+      const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+      // Lazy rescale: move this row's reference max only when it grows by > 2^8.
+      const bool grow = valid && (m_run == -INFINITY ? mx != -INFINITY : mx > m_run + kRescaleThreshold);
+      const bool rescale_o = grow && m_run != -INFINITY;
+      any_rescale = __any_sync(0xffffffffu, rescale_o);
+      alpha = rescale_o ? ex2(m_run - mx) : 1.f;
+      l_run *= alpha;
+      if (grow) m_run = mx;
+      const float m_use = m_run == -INFINITY ? 0.f : m_run;
+      float ps4[4] = {0.f, 0.f, 0.f, 0.f};
+      uint32_t pk[kTileKeys / 2];  // P as bf16 pairs (rows past the stack hold zeros)
+#pragma unroll
+      for (int k = 0; k < kTileKeys / 2; ++k) {
+        const float e0 = ex2(pr[2 * k] - m_use), e1 = ex2(pr[2 * k + 1] - m_use);
+        ps4[(2 * k) & 3] += e0;
+        ps4[(2 * k + 1) & 3] += e1;
+        pk[k] = pack_bf16x2(e0, e1);
+      }
+      l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
+      tmem_st32(my_s + j * kTileKeys, pk);  // P over the S columns just read
+    }
+    // P.V of the previous tile must complete before P of this tile is released: O_wg may then be
+    // rescaled, and pvdone never runs two phases ahead of this warpgroup's waits (P.V of tile t needs
+    // the pfull below; S of this tile implies P.V of tile t - 2), so its parity stays unambiguous.
+    if (live && t > 0 && !mbar_wait(smem_addr(&sm.pvdone[wg]), (t - 1) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
+    if (live && warp_live) {
+      if (any_rescale) {  // O_wg *= alpha (P.V of this tile is issued only after pfull below)
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[32];
+          tmem_ld32(my_o + 32 * c, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * alpha);
+          tmem_st32(my_o + 32 * c, o);
+        }
+      }
+      tmem_wait_st();
+    }
+    if (wg == 0 && live && ti.nkeys < kTileKeys) {
+      // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.  Warpgroup 0 clears them
+      // before it releases P_0, and both P.V of the tile are issued after P_0's.
+      if (!mbar_wait(smem_addr(&sm.vfull[t % kPairNV]), (t / kPairNV) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
+      uint8_t* vptr = sm.vring + static_cast<size_t>(t % kPairNV) * kKVBytes;
+      const bool grouped = ti.draft || p.prefix_grouped;
+      const int nz = (kTileKeys - ti.nkeys) * 16;
+      for (int i = wtid; i < nz; i += kQRows) {
+        const int key = ti.nkeys + (i >> 4), ch = i & 15;
+        *reinterpret_cast<uint4*>(vptr + tile_off_tc(key, ch, grouped)) = make_uint4(0, 0, 0, 0);
+      }
+      fence_proxy_async_smem();
+    }
+    tc_fence_before();
+    mbar_arrive(smem_addr(&sm.pfull[2 * wg + j]));
+    if (ti.last) {
+      // Every P.V of the piece has completed once P.V of tile t has (P.V of tile t - 1 was waited above).
+      bool ok = live && mbar_wait(smem_addr(&sm.pvdone[wg]), t & 1, p.err, p.wait_ns);
+      ok = __all_sync(0xffffffffu, ok);
+      tc_fence_after();
+      if (ok && warp_live) {
+        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+        const float lse2 = l_run > 0.f ? m_run + __log2f(l_run) : -INFINITY;
+        const bool whole = cu.lt == cu.ut - 1 && (cu.t - cu.t_begin) >= cu.lt;
+        const int slot = cu.c * HR + cu.hr + blockIdx.x;
+        const int urow = wg * kQRows + r;  // row within the unit
+        size_t orow = 0;
+        if (valid && whole) {
+          const int g = rr - nl * p.G;
+          orow = (static_cast<size_t>(cu.c) * p.Nq + nl) * p.hq + h * p.G + g;
+        }
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[32];
+          tmem_ld32(my_o + 32 * c, o);
+          tmem_wait_ld();
+          if (valid) {
+            if (whole) {
+              uint4* dst = reinterpret_cast<uint4*>(p.out + orow * kHeadDim + 32 * c);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                uint4 w4;
+                w4.x = pack_bf16x2(__uint_as_float(o[8 * k + 0]) * inv, __uint_as_float(o[8 * k + 1]) * inv);
+                w4.y = pack_bf16x2(__uint_as_float(o[8 * k + 2]) * inv, __uint_as_float(o[8 * k + 3]) * inv);
+                w4.z = pack_bf16x2(__uint_as_float(o[8 * k + 4]) * inv, __uint_as_float(o[8 * k + 5]) * inv);
+                w4.w = pack_bf16x2(__uint_as_float(o[8 * k + 6]) * inv, __uint_as_float(o[8 * k + 7]) * inv);
+                dst[k] = w4;
+              }
+            } else {
+              float4* dst = reinterpret_cast<float4*>(
+                  p.ws_o + (static_cast<size_t>(slot) * p.rows_per_unit + urow) * kHeadDim + 32 * c);
+#pragma unroll
+              for (int k = 0; k < 8; ++k)
+                dst[k] = make_float4(__uint_as_float(o[4 * k]) * inv, __uint_as_float(o[4 * k + 1]) * inv,
+                                     __uint_as_float(o[4 * k + 2]) * inv, __uint_as_float(o[4 * k + 3]) * inv);
+            }
+          }
+        }
+        if (valid) {
+          if (whole) p.lse[orow] = lse2 * 0.69314718055994531f;
+          else p.ws_lse[static_cast<size_t>(slot) * p.rows_per_unit + urow] = lse2;
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(smem_addr(&sm.ofree[wg]));
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_tc_pair_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ TensorMaps maps, int nq_box) {
+  extern __shared__ uint8_t smem_raw[];
+  if (threadIdx.x == 0) allow_dependent_launch();  // the merge may be scheduled as CTAs finish
+  const int len0 = static_cast<int>(threadIdx.x) < p.C ? p.seq_lens[threadIdx.x] : -1;
+  const SmemPair sm = carve_pair(smem_raw, p.C);
+  const int warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kPairNK; ++s) {
+      mbar_init(smem_addr(&sm.kfull[s]), 1);
+      mbar_init(smem_addr(&sm.kempty[s]), 1);
+    }
+    for (int s = 0; s < kPairNV; ++s) {
+      mbar_init(smem_addr(&sm.vfull[s]), 1);
+      mbar_init(smem_addr(&sm.vempty[s]), 1);
+    }
+    mbar_init(smem_addr(sm.qfull), 1);
+    mbar_init(smem_addr(sm.qempty), 1);
+    for (int b = 0; b < 4; ++b) {
+      mbar_init(smem_addr(&sm.sfull[b]), 1);
+      mbar_init(smem_addr(&sm.sfree[b]), 1);
+      mbar_init(smem_addr(&sm.pfull[b]), kQRows);
+    }
+    for (int w = 0; w < 2; ++w) {
+      mbar_init(smem_addr(&sm.pvdone[w]), 1);
+      mbar_init(smem_addr(&sm.ofree[w]), kQRows);
+      mbar_init(smem_addr(&sm.mmadone[w]), 1);
+    }
+    for (int i = 0; i < kMiscInts; ++i) sm.misc[i] = 0;
+    fence_mbar_init();
+    prefetch_tensormap(&maps.tk);
+    prefetch_tensormap(&maps.tv);
+    prefetch_tensormap(&maps.dk);
+    prefetch_tensormap(&maps.dv);
+    prefetch_tensormap(&maps.q);
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_addr(sm.tmem_base), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  build_plan(p, sm.len, sm.base, len0);  // block-wide barriers inside
+  tc_fence_after();
+  const uint32_t tmem = *sm.tmem_base;
+  const Cursor cu = cursor_begin(p, sm.len, sm.base);
+  Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), nullptr};
+  if (warp == kProducerWarp || warp == kProducerVWarp) {
+    run_producer_tc<kModePair>(p, maps, sm, pipe, cu, nq_box, warp == kProducerWarp ? 0 : 1);
+  } else if (warp == kMmaWarp || warp == kMmaPvWarp) {
+    const int stream = warp == kMmaWarp ? 0 : 1;
+    if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
+      if (stream == 0) run_mma_qk_pair(p, sm, pipe, tmem, cu);
+      else run_mma_pv_pair(p, sm, pipe, tmem, cu);
+      // Every MMA must have completed before TMEM is released (retried, bounded, as in attn_tc_kernel).
+      for (int k = 0; k < 4 && !mbar_wait(smem_addr(&sm.mmadone[stream]), 0, p.err); ++k) {
+      }
+    }
+    __syncwarp();
+  } else if (warp < 8) {
+    run_softmax_pair(p, sm, pipe, tmem, cu);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (threadIdx.x == 0 && *pipe.abort) {
+    // A wait timed out: let every TMA load still in flight land before the CTA exits.
+    for (int k = sm.misc[2]; k < max(sm.misc[8], sm.misc[9]); ++k)
+      if (k < sm.misc[8 + (k & 1)] && !mbar_wait(smem_addr(&sm.kfull[k % kPairNK]), (k / kPairNK) & 1, p.err)) break;
+    for (int k = sm.misc[6]; k < max(sm.misc[10], sm.misc[11]); ++k)
+      if (k < sm.misc[10 + (k & 1)] && !mbar_wait(smem_addr(&sm.vfull[k % kPairNV]), (k / kPairNV) & 1, p.err)) break;
+    for (int k = sm.misc[4]; k < sm.misc[3]; ++k)
+      if (!mbar_wait(smem_addr(sm.qfull), k & 1, p.err)) break;
+  }
+  if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
 }
 
 template <bool kSpread>
@@ -761,7 +1246,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const Cursor cu = cursor_begin(p, sm.len, sm.base);
   Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), nullptr};
   if (warp == kProducerWarp || warp == kProducerVWarp) {
-    run_producer_tc<kSpread>(p, maps, sm, pipe, cu, nq_box, warp == kProducerWarp ? 0 : 1);
+    run_producer_tc<kSpread ? kModeSpread : kModeDense>(p, maps, sm, pipe, cu, nq_box, warp == kProducerWarp ? 0 : 1);
   } else if (warp == kMmaWarp || warp == kMmaPvWarp) {
     const int stream = warp == kMmaWarp ? 0 : 1;
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
@@ -803,8 +1288,16 @@ cudaError_t attn_tc_occupancy(int C, int* ctas_per_sm) {
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, attn_tc_kernel<false>, kThreads, smem);
 }
 
-cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, bool pdl,
+cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, bool pair, bool pdl,
                            cudaStream_t stream) {
+  if (pair) {
+    const size_t smem = smem_bytes_pair(p.C);
+    cudaError_t e = cudaFuncSetAttribute(attn_tc_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    return launch_maybe_pdl(attn_tc_pair_kernel, dim3(p.num_ctas), dim3(kThreads), smem, pdl, stream, p, maps,
+                            nq_box);
+  }
   const size_t smem = smem_bytes(p.C);
   auto* kernel = spread ? attn_tc_kernel<true> : attn_tc_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));

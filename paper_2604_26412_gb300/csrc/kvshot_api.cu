@@ -146,6 +146,7 @@ struct Plan {
   int m_tiles;        // mma path
   int nq_box;         // tensor-memory path: draft nodes per 128-row block
   bool spread;        // tensor-memory path: 16 rows per TMEM lane quarter
+  bool pair;          // tensor-memory path: two 128-row blocks per unit (stacks of more than 128 rows)
   int rows_per_unit;
   int row_blocks;
   int units;
@@ -235,6 +236,7 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   pl->m_tiles = 0;
   pl->nq_box = 0;
   pl->spread = false;
+  pl->pair = false;
   if (pl->kernel == Kernel::kMma) {
     pl->m_tiles = std::min(kMmaMaxTiles, std::max(1, (rows + 15) / 16));
     pl->rows_per_unit = 16 * pl->m_tiles;
@@ -242,6 +244,9 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
     pl->nq_box = std::max(1, std::min(d->n_query, 128 / G));
     pl->rows_per_unit = G * pl->nq_box;
     pl->spread = pl->rows_per_unit <= kSpreadMaxRows;
+    // More than 128 rows: each unit takes two 128-row blocks, so every K/V tile feeds both.
+    pl->pair = rows > 128;
+    if (pl->pair) pl->rows_per_unit = 2 * 128;
   } else {
     pl->rows_per_unit = kCcRows;
   }
@@ -410,7 +415,7 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const bool pdl = (d->flags & KVSHOT_OVERLAP_PREVIOUS) != 0;
   cudaError_t e = pl.kernel == Kernel::kMma            ? launch_attn_mma(p, maps, pl.m_tiles, pdl, s)
-                  : pl.kernel == Kernel::kTensorMemory ? launch_attn_tc(p, maps, pl.nq_box, pl.spread, pdl, s)
+                  : pl.kernel == Kernel::kTensorMemory ? launch_attn_tc(p, maps, pl.nq_box, pl.spread, pl.pair, pdl, s)
                                                        : launch_attn_cc(p, maps, pdl, s);
   if (e != cudaSuccess) return KVSHOT_ERR_CUDA;
   e = launch_merge(p, s);

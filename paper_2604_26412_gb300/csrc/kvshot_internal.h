@@ -117,7 +117,7 @@ bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t 
 // launch with programmatic stream serialization (KVSHOT_OVERLAP_PREVIOUS).
 cudaError_t launch_attn_cc(const AttnParams& p, const TensorMaps& maps, bool pdl, cudaStream_t stream);
 cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, bool pdl, cudaStream_t stream);
-cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, bool pdl,
+cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, bool pair, bool pdl,
                            cudaStream_t stream);
 
 // Launches `kernel` on grid x block with `smem` dynamic bytes; with programmatic stream

@@ -72,6 +72,11 @@ CASES = [
     ((600, 129), (8, 12), True, True, 16, 32, 8, 20),             # 80 rows: dense TMEM rows, partial quarter
     ((300,), (2, 2), True, False, 16, 32, 2, 3),                  # G = 16: 48 rows spread, boxes of one node
     ((250, 70), (1, 1, 1), False, True, 16, 32, 1, 2),            # G = 32: 64 rows spread, boxes of 16 heads
+    ((257, 513, 0), (8, 12, 12, 12), True, True, 16, 32, 8, 40),  # 160 rows: paired blocks, block 1 mostly empty
+    ((1, 64, 130), (8, 12, 12, 12, 12, 8), True, True, 16, 32, 8, 64),  # 256 rows paired, ragged prefixes
+    ((203,), tuple([1] * 40), False, False, 16, 32, 8, 40),       # whole chain: paired, contiguous l_cap % 8 != 0
+    ((96, 200), tuple([1] * 100), False, True, 16, 32, 8, 100),   # 400 rows: two paired units per KV head
+    ((500,), (4, 8, 8), True, True, 64, 64, 8, 20),               # G = 8: 160 rows paired, 64-token pages
 ]
 
 

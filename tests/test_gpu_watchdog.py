@@ -6,7 +6,7 @@ yet: the call must still end (the abort drains the copies and tensor-core
 operations already issued, with the ordinary 2 s limit), record
 KVSHOT_ERR_TIMEOUT in err_flag, and leave the stream, the device and the
 workspace fit for the next call, which must match the CPU oracle.  Every
-kernel is driven through its abort path: tcgen05 with spread and dense rows,
+kernel is driven through its abort path: tcgen05 with spread, dense and paired rows,
 m16n8k16 and the CUDA-core kernel.
 """
 import pytest
@@ -20,7 +20,7 @@ pytestmark = pytest.mark.gpu
 
 
 def _problem(n_query, seed):
-    spec = wl.Spec("watchdog", 3, 1, [3000, 517, 64], [8, 12, 12], True, True, page_size=16, seed=seed)
+    spec = wl.Spec("watchdog", 3, 1, [3000, 517, 64], [8, 12, 12, 12], True, True, page_size=16, seed=seed)
     inp = wl.make_inputs(spec, "cuda", seed=seed, tail_fill="nan")
     N = spec.n_nodes
     dk, dv = wl.random_draft_kv(spec, inp.n_max, N, "cuda", seed=seed + 1)
@@ -50,6 +50,7 @@ def _call(spec, inp, dk, dv, q, N, flags, wait_limit_ns, ws):
 @pytest.mark.parametrize("flags,n_query", [
     (kvshot.KVSHOT_FORCE_TC, 12),    # 48 rows: spread TMEM rows
     (kvshot.KVSHOT_FORCE_TC, 32),    # 128 rows: dense TMEM rows
+    (kvshot.KVSHOT_FORCE_TC, 40),    # 160 rows: paired row blocks
     (kvshot.KVSHOT_FORCE_MMA, 4),
     (kvshot.KVSHOT_FORCE_CC, 4),
 ])
