@@ -36,11 +36,11 @@ namespace {
 using namespace dev;
 using namespace tc;
 
-constexpr int kNK = 4;                     // K tiles in flight (freed when QK^T completes)
-constexpr int kNV = 5;                     // V tiles in flight (freed when P.V completes)
+constexpr int kNK = 5;                     // K tiles in flight (freed when QK^T completes)
+constexpr int kNV = 6;                     // V tiles in flight (freed when P.V completes)
 constexpr int kKVBytes = kKVTileBytes;     // one K or V tile
 constexpr int kNS = 4;                     // S buffers in TMEM: QK^T may run up to 4 tiles ahead of P.V
-constexpr int kNP = 2;                     // P buffers in shared memory (buffer w: warpgroup w's tiles)
+constexpr int kNW = 2;                     // O accumulators: warpgroup w's tiles accumulate into O_w
 constexpr int kThreads = 12 * 32;
 constexpr int kProducerWarp = 10;          // K and V loads of even tiles
 constexpr int kProducerVWarp = 9;          // K and V loads of odd tiles, q blocks
@@ -48,7 +48,6 @@ constexpr int kMmaWarp = 11;               // TMEM owner, QK^T issuer
 constexpr int kMmaPvWarp = 8;              // P.V issuer
 constexpr int kSoftmaxThreads = 256;       // two warpgroups
 constexpr int kBarSoftmax = 1;             // named barrier among the softmax warps
-constexpr int kPBufBytes = kQRows * 128;   // 128 rows x 64 keys bf16
 constexpr uint32_t kTmemCols = 512;        // S0..S3 [0,256), O0 [256,384), O1 [384,512)
 constexpr uint32_t kTmemO = kNS * kTileKeys;
 constexpr int kMiscInts = 12;
@@ -80,16 +79,16 @@ struct Smem {
   uint8_t* kring;      // kNK x K tile
   uint8_t* vring;      // kNV x V tile
   uint8_t* qbuf;       // one q block
-  uint8_t* pbuf;       // kNP x kPBufBytes
-  uint64_t* kfull;     // [kNK]  TMA -> MMA (a K slot is free again once QK^T of its tile completed: sfull)
+  uint64_t* kfull;     // [kNK]  TMA -> MMA
+  uint64_t* kempty;    // [kNK]  QK^T of the slot's tile completed -> TMA
   uint64_t* vfull;     // [kNV]  TMA -> MMA, softmax
   uint64_t* vempty;    // [kNV]  P.V completion -> TMA
   uint64_t* qfull;     // [1]
   uint64_t* qempty;    // [1]
   uint64_t* sfull;     // [kNS]  S buffer written (QK^T completion)
-  uint64_t* sfree;     // [kNS]  S buffer read (the owning warpgroup's 128 threads)
-  uint64_t* pfull;     // [kNP]  P buffer written and S consumed (256 softmax threads)
-  uint64_t* pvdone;    // [kNP]  P.V of the tile using that buffer completed
+  uint64_t* sfree;     // [kNS]  P.V of the tile in the S buffer completed: the buffer is free
+  uint64_t* pfull;     // [kNS]  P written over the S buffer (the owning warpgroup's 128 threads)
+  uint64_t* pvdone;    // [kNW]  P.V into O_w of warpgroup w's latest tile completed
   uint64_t* ofree;     // [1]  epilogue finished reading O
   uint64_t* mmadone;   // [2]  every QK^T / every P.V completed
   uint64_t* anc;       // [64]
@@ -103,8 +102,8 @@ struct Smem {
 };
 
 __host__ __device__ inline size_t smem_bytes(int C) {
-  size_t off = static_cast<size_t>(kNK + kNV) * kKVBytes + kQBufBytes + kNP * kPBufBytes;
-  off += sizeof(uint64_t) * (kNK + 2 * kNV + 2 + 2 * kNS + 2 * kNP + 3);
+  size_t off = static_cast<size_t>(kNK + kNV) * kKVBytes + kQBufBytes;
+  off += sizeof(uint64_t) * (2 * kNK + 2 * kNV + 2 + 3 * kNS + kNW + 3);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(float) * 2 * kQRows;
   off += sizeof(uint32_t) * 4 + sizeof(int) * kMiscInts;
@@ -121,19 +120,18 @@ __device__ Smem carve(uint8_t* raw, int C) {
   p += kNV * kKVBytes;
   s.qbuf = p;
   p += kQBufBytes;
-  s.pbuf = p;
-  p += kNP * kPBufBytes;
   uint64_t* b = reinterpret_cast<uint64_t*>(p);
   s.kfull = b;
-  s.vfull = s.kfull + kNK;
+  s.kempty = s.kfull + kNK;
+  s.vfull = s.kempty + kNK;
   s.vempty = s.vfull + kNV;
   s.qfull = s.vempty + kNV;
   s.qempty = s.qfull + 1;
   s.sfull = s.qempty + 1;
   s.sfree = s.sfull + kNS;
   s.pfull = s.sfree + kNS;
-  s.pvdone = s.pfull + kNP;
-  s.ofree = s.pvdone + kNP;
+  s.pvdone = s.pfull + kNS;
+  s.ofree = s.pvdone + kNW;
   s.mmadone = s.ofree + 1;
   s.anc = s.mmadone + 2;
   s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
@@ -152,8 +150,9 @@ __device__ Smem carve(uint8_t* raw, int C) {
 // QK^T in tile order from warp kMmaWarp, P.V in tile order from warp
 // kMmaPvWarp.  A tcgen05.commit tracks the MMAs of the thread that issues it.
 
-// S = Q K^T of every tile.  Tile t needs its K tile, its S buffer read by the
-// softmax of tile t - kNS, and (first tile of a piece) the piece's q block.
+// S = Q K^T of every tile.  Tile t needs its K tile, its S buffer freed by
+// the completion of P.V of tile t - kNS, and (first tile of a piece) the
+// piece's q block.
 __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                            Cursor cu) {
   constexpr uint32_t idesc = idesc_bf16(128, 64, false);
@@ -184,14 +183,17 @@ __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, 
       tc_mma(tmem + (t % kNS) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
     }
     tc_commit(smem_addr(&sm.sfull[t % kNS]));
+    tc_commit(smem_addr(&sm.kempty[t % kNK]));
     if (ti.last) tc_commit(smem_addr(sm.qempty));
   }
   tc_commit(smem_addr(&sm.mmadone[0]));
 }
 
-// O_w += P V of every tile, w = t % 2 (the warpgroup that wrote P).  Tile t
-// needs its P and its V tile; the first P.V into O_w of a piece (which
-// overwrites O_w) needs the previous piece's epilogue to have read O.
+// O_w += P V of every tile, w = t % 2 (the warpgroup that wrote P), with P
+// read from tensor memory (the tile's S columns).  Tile t needs its P and its
+// V tile; the first P.V into O_w of a piece (which overwrites O_w) needs the
+// previous piece's epilogue to have read O.  Each completion frees the tile's
+// S buffer for QK^T of tile t + kNS.
 __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                            Cursor cu) {
   constexpr uint32_t idesc = idesc_bf16(128, 128, true);
@@ -205,7 +207,7 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
     const bool first = t - piece_t0 < 2;
     bool ok = !*pipe.abort;
     if (ok && first && piece > 1) ok = mbar_wait(smem_addr(sm.ofree), (piece - 2) & 1, p.err, p.wait_ns);
-    if (ok) ok = mbar_wait(smem_addr(&sm.pfull[t % kNP]), (t / kNP) & 1, p.err, p.wait_ns);
+    if (ok) ok = mbar_wait(smem_addr(&sm.pfull[t % kNS]), (t / kNS) & 1, p.err, p.wait_ns);
     if (ok) ok = mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err, p.wait_ns);
     if (!ok) {
       *pipe.abort = 1;
@@ -213,20 +215,20 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
     }
     sm.misc[6] = t + 1;
     tc_fence_after();
-    const uint32_t pbase = smem_addr(sm.pbuf + (t % kNP) * kPBufBytes);
+    const uint32_t pcol = tmem + (t % kNS) * kTileKeys;  // P: 32 columns of bf16 pairs
     const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(t % kNV) * kKVBytes);
     const uint32_t o = tmem + kTmemO + 128 * (t & 1);
     const bool grouped = ti.draft || p.prefix_grouped;
     const uint32_t half_off = grouped ? kGroupHalfBytes : kHalfBytes, group_off = grouped ? kGroupBytes : 1024;
 #pragma unroll
     for (int k16 = 0; k16 < kTileKeys / 16; ++k16) {  // 16-key steps of the tile
-      const uint64_t a = smem_desc_sw128(pbase + k16 * 32, 16, 1024);
       // V tile is MN-major: 64-dim halves `half_off` apart (leading), 8-key groups `group_off` apart (stride).
       const uint64_t bd = smem_desc_sw128(vbase + k16 * 2 * group_off, half_off, group_off);
-      tc_mma(o, a, bd, idesc, (first && k16 == 0) ? 0u : 1u);
+      tc_mma_tmem_a(o, pcol + 8 * k16, bd, idesc, (first && k16 == 0) ? 0u : 1u);
     }
     tc_commit(smem_addr(&sm.vempty[t % kNV]));
-    tc_commit(smem_addr(&sm.pvdone[t % kNP]));
+    tc_commit(smem_addr(&sm.pvdone[t & 1]));
+    tc_commit(smem_addr(&sm.sfree[t % kNS]));
   }
   tc_commit(smem_addr(&sm.mmadone[1]));
 }
@@ -248,7 +250,7 @@ template <bool kSpread>
 __device__ __forceinline__ void rescale_o_tmem(const Smem& sm, const Pipe& pipe, const AttnParams& p, uint32_t my_o,
                                                int t, float alpha) {
   constexpr int kOChunks = kSpread ? 2 : 4;  // 32-column O chunks per thread
-  if (!mbar_wait(smem_addr(&sm.pvdone[(t - 2) % kNP]), ((t - 2) / kNP) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
+  if (!mbar_wait(smem_addr(&sm.pvdone[t & 1]), ((t - 2) / kNW) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
   tc_fence_after();
 #pragma unroll
   for (int c = 0; c < kOChunks; ++c) {
@@ -320,7 +322,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
     }
     bool live = !*pipe.abort;
     if ((t & 1) == wg) {
-      const int sbuf = t % kNS, b = t % kNP;
+      const int sbuf = t % kNS;
       if (live && !mbar_wait(smem_addr(&sm.sfull[sbuf]), (t / kNS) & 1, p.err, p.wait_ns)) {
         *pipe.abort = 1;
         live = false;
@@ -330,7 +332,6 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       float pr[kCols];
       bool any_rescale = false;  // dense rows: some row of this warp moves its reference max, O_wg is rescaled
       float alpha = 1.f;         // dense rows: this row's factor
-      if (!(live && warp_live)) mbar_arrive(smem_addr(&sm.sfree[sbuf]));  // S is not read
       if (live && warp_live) {
         uint32_t sv[kCols];
         if constexpr (kSpread) {
@@ -340,8 +341,6 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
           tmem_ld32(trow + sbuf * kTileKeys + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
         }
         tmem_wait_ld();
-        tc_fence_before();
-        mbar_arrive(smem_addr(&sm.sfree[sbuf]));
         // Visible keys of this row (bit j = key key0 + j).
         uint64_t v64 = 0;
         if (valid) {
@@ -396,31 +395,27 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         if (grow) m_run = mx;
         const float m_use = m_run == -INFINITY ? 0.f : m_run;
         float ps4[4] = {0.f, 0.f, 0.f, 0.f};
+        uint32_t pk[kCols / 2];  // P as bf16 pairs over the S columns just read (rows past the stack: zeros)
 #pragma unroll
-        for (int j = 0; j < kCols; ++j) {
-          pr[j] = ex2(pr[j] - m_use);
-          ps4[j & 3] += pr[j];
+        for (int j = 0; j < kCols / 2; ++j) {
+          const float e0 = ex2(pr[2 * j] - m_use), e1 = ex2(pr[2 * j + 1] - m_use);
+          ps4[(2 * j) & 3] += e0;
+          ps4[(2 * j + 1) & 3] += e1;
+          pk[j] = pack_bf16x2(e0, e1);
         }
         l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
+        if constexpr (kSpread) tmem_st16x2_16(trow + sbuf * kTileKeys, pk);
+        else tmem_st32(trow + sbuf * kTileKeys, pk);
       }
-      // The P buffer is free once P.V of tile t - kNP has completed.
-      if (live && t >= kNP && !mbar_wait(smem_addr(&sm.pvdone[b]), ((t - kNP) / kNP) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
-      if (live && valid) {
-        uint8_t* prow = sm.pbuf + b * kPBufBytes + tl * 128;
-#pragma unroll
-        for (int c = 0; c < kCols / 8; ++c) {
-          const int chunk = (col0 >> 3) + c;  // 16-byte chunk = 8 keys
-          uint4 w;
-          w.x = pack_bf16x2(pr[8 * c + 0], pr[8 * c + 1]);
-          w.y = pack_bf16x2(pr[8 * c + 2], pr[8 * c + 3]);
-          w.z = pack_bf16x2(pr[8 * c + 4], pr[8 * c + 5]);
-          w.w = pack_bf16x2(pr[8 * c + 6], pr[8 * c + 7]);
-          *reinterpret_cast<uint4*>(prow + ((chunk ^ (tl & 7)) << 4)) = w;
-        }
-      }
+      // P.V of this warpgroup's previous tile must complete before P of this tile is released: O_wg may
+      // then be rescaled, and pvdone never runs two phases ahead of this warpgroup's waits (S of this tile
+      // implies P.V of tile t - kNS; P.V of tile t needs the pfull below).
+      if (live && t >= kNW && !mbar_wait(smem_addr(&sm.pvdone[t & 1]), ((t - kNW) / kNW) & 1, p.err, p.wait_ns))
+        *pipe.abort = 1;
       if constexpr (!kSpread) {
         if (live && warp_live && any_rescale) rescale_o_tmem<kSpread>(sm, pipe, p, my_o, t, alpha);
       }
+      if (live && warp_live) tmem_wait_st();
       if (live && ti.nkeys < kTileKeys) {
         // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.
         if (!mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
@@ -433,7 +428,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       }
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(smem_addr(&sm.pfull[b]));
+      mbar_arrive(smem_addr(&sm.pfull[sbuf]));
     }
     if (ti.last) {
       // Every P.V of the piece has completed once P.V of tile t has (P.V
@@ -442,8 +437,8 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       // from tile t - 6's by parity, so it first waits P.V of its own tile t - 1.
       bool ok = live;
       if (ok && (t & 1) != wg && t >= 1)
-        ok = mbar_wait(smem_addr(&sm.pvdone[(t - 1) % kNP]), ((t - 1) / kNP) & 1, p.err, p.wait_ns);
-      ok = ok && mbar_wait(smem_addr(&sm.pvdone[t % kNP]), (t / kNP) & 1, p.err, p.wait_ns);
+        ok = mbar_wait(smem_addr(&sm.pvdone[(t - 1) & 1]), ((t - 1) / kNW) & 1, p.err, p.wait_ns);
+      ok = ok && mbar_wait(smem_addr(&sm.pvdone[t & 1]), (t / kNW) & 1, p.err, p.wait_ns);
       ok = __all_sync(0xffffffffu, ok);
       tc_fence_after();
       float l_row = l_run;
@@ -693,25 +688,13 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
     const int kv = lane >> 4, i = lane & 15;
     const int kslot = t % NK, vslot = t % NV;
     // A V slot is free once P.V of its previous tile completed, a K slot once QK^T of its previous tile
-    // (t - NK) completed.  Lane 0 waits for the K slot and lane 1 for the V slot together.  Single
-    // blocks read the K-slot release off the S buffer of tile t - NK, whose next completion (tile t)
-    // needs this very K tile, so its phase cannot be mistaken for one two phases later.  Paired blocks
-    // have only two S buffers per block (tile t - NK + 2 < t may complete first), so their K slots
-    // have release barriers of their own.
+    // (t - NK) completed; each slot has its own release barrier, whose next completion (tile t) needs
+    // this very load, so a phase is never mistaken for one two phases later.  Lane 0 waits for the K
+    // slot and lane 1 for the V slot together.
     if (lane < 2 && ok) {
-      const bool need = lane == 1 || t >= NK || kMode == kModePair;
-      const int tk = t - NK;
-      uint32_t kbar, kpar;
-      if constexpr (kMode == kModePair) {
-        kbar = smem_addr(&sm.kempty[kslot]);
-        kpar = ((t / NK) & 1) ^ 1u;
-      } else {
-        kbar = smem_addr(&sm.sfull[tk % kNS]);
-        kpar = (tk / kNS) & 1;
-      }
-      const uint32_t bar = lane == 0 ? kbar : smem_addr(&sm.vempty[vslot]);
-      const uint32_t par = lane == 0 ? kpar : (((t / NV) & 1) ^ 1u);
-      ok = (!need || mbar_wait(bar, par, p.err, p.wait_ns)) && !*pipe.abort;
+      const uint32_t bar = lane == 0 ? smem_addr(&sm.kempty[kslot]) : smem_addr(&sm.vempty[vslot]);
+      const uint32_t par = ((t / (lane == 0 ? NK : NV)) & 1) ^ 1u;
+      ok = mbar_wait(bar, par, p.err, p.wait_ns) && !*pipe.abort;
     }
     ok = __all_sync(0xffffffffu, ok);
     if (!ok) {
@@ -1209,7 +1192,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       asm volatile("prefetch.global.L2 [%0];" ::"l"(p.page_table + c * p.max_pages + pg));
   }
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kNK; ++s) mbar_init(smem_addr(&sm.kfull[s]), 1);
+    for (int s = 0; s < kNK; ++s) {
+      mbar_init(smem_addr(&sm.kfull[s]), 1);
+      mbar_init(smem_addr(&sm.kempty[s]), 1);
+    }
     for (int s = 0; s < kNV; ++s) {
       mbar_init(smem_addr(&sm.vfull[s]), 1);
       mbar_init(smem_addr(&sm.vempty[s]), 1);
@@ -1218,12 +1204,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(smem_addr(sm.qempty), 1);
     for (int b = 0; b < kNS; ++b) {
       mbar_init(smem_addr(&sm.sfull[b]), 1);
-      mbar_init(smem_addr(&sm.sfree[b]), kSoftmaxThreads / 2);
-    }
-    for (int b = 0; b < kNP; ++b) {
+      mbar_init(smem_addr(&sm.sfree[b]), 1);
       mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads / 2);
-      mbar_init(smem_addr(&sm.pvdone[b]), 1);
     }
+    for (int w = 0; w < kNW; ++w) mbar_init(smem_addr(&sm.pvdone[w]), 1);
     mbar_init(smem_addr(sm.ofree), kSoftmaxThreads);
     mbar_init(smem_addr(&sm.mmadone[0]), 1);
     mbar_init(smem_addr(&sm.mmadone[1]), 1);
