@@ -785,6 +785,30 @@ def run_project(args, world, rank, local):
             b.record(stream)
     torch.cuda.synchronize()
     call_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    # Launch floor: the same two-kernel call on 1 token, 1 layer and 1 KV head (fixed costs only).
+    fl_in = wl.project_inputs(1, 1, 1, device="cuda", seed=args.seed + 9)
+    fl_pool = torch.zeros((P, wl.HEAD_DIM), dtype=torch.bfloat16, device="cuda")
+    fl_pt = torch.zeros((1, 1), dtype=torch.int32, device="cuda")
+    fl_desc = kvshot.make_project_desc(num_tokens=1, num_layers=1, hkv=1, num_caches=1, page_size=P,
+                                       max_pages_per_seq=1, num_pages=1, rope_base=spec.rope_base, rope=True,
+                                       err_flag=err)
+    fl_ws = torch.empty(max(256, kvshot.kv_project_workspace_size(fl_desc)), dtype=torch.uint8, device="cuda")
+    fl_desc.workspace, fl_desc.workspace_bytes = fl_ws.data_ptr(), fl_ws.numel()
+    fl_tc = torch.zeros(1, dtype=torch.int32, device="cuda")
+    fl_v = torch.zeros_like(fl_pool)
+    fl_call = lambda: kvshot.kv_project(fl_desc, fl_in.k_in, fl_in.v_in, fl_in.w_k, fl_in.w_v, fl_tc, fl_tc, fl_pt,
+                                        fl_pool, fl_v, stream)
+    ev_fl = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            fl_call()
+        torch.cuda._sleep(int(2e7))
+        for a, b in ev_fl:
+            a.record(stream)
+            fl_call()
+            b.record(stream)
+    torch.cuda.synchronize()
+    floor_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_fl)
     nbytes = project_bytes(T, L, dkv)
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
@@ -792,7 +816,9 @@ def run_project(args, world, rank, local):
     roofline = {"bound": "hbm", "kernel": "kvshot_kv_project (tcgen05 slab GEMM + RoPE/store kernels)",
                 "achieved": round(achieved, 1), "peak": hbm_peak, "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
                 "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback 6.8 TB/s",
-                "traffic": None, "algorithmic_bytes_per_call": nbytes, "call_us": round(call_ms * 1e3, 2)}
+                "traffic": None, "algorithmic_bytes_per_call": nbytes, "call_us": round(call_ms * 1e3, 2),
+                "launch_floor_us": round(floor_ms * 1e3, 2),
+                "launch_floor": "the same call on 1 token x 1 layer x 1 KV head (both kernels' fixed costs)"}
     k_h, v_h = pi.k_in.cpu().pin_memory(), pi.v_in.cpu().pin_memory()
     k_d, v_d = torch.empty_like(pi.k_in), torch.empty_like(pi.v_in)
     e2e_steps = max(3, min(args.steps, 100))

@@ -16,9 +16,12 @@
 // Two kernels.  The slab GEMM (kvshot_slab_gemm.cuh) computes the products per
 // layer block (table entry (K or V, layer l): W[:, l d_kv : (l+1) d_kv] times
 // the tokens' layer-l K or V), into fp32 slabs [2 L_s][T][d_kv].
-// kv_project_finish adds each output's L_s slabs, rotates the keys (angles in
-// fp64 from a host table of rope_base^(-2j/128)), rounds to bf16 and stores
-// both vectors into the cache through the page table.
+// kv_project_finish adds each output's L_s slabs, rotates the keys, rounds to
+// bf16 and stores both vectors into the cache through the page table.  The
+// angle pos * rope_base^(-2j/128) is formed and reduced modulo 2 pi in fp64
+// (from a host table of the frequencies); sine, cosine and the rotation are
+// fp32 (relative error ~1e-7, far below the bf16 rounding that follows).
+// fp64 sine and cosine cost this latency-bound kernel ~2 us per call on GB300.
 #include <algorithm>
 #include <cmath>
 
@@ -81,11 +84,13 @@ __global__ void __launch_bounds__(kFinishThreads) kv_project_finish(const __grid
     vy += p.slab[(p.L + l) * td + f + 64];
   }
   if (p.rope) {
-    double sn, cs;
-    sincos(static_cast<double>(pos) * p.inv_freq[j], &sn, &cs);
-    const double x = kx, y = ky;
-    kx = static_cast<float>(x * cs - y * sn);
-    ky = static_cast<float>(y * cs + x * sn);
+    const double a = static_cast<double>(pos) * p.inv_freq[j];
+    const double r = a - 6.283185307179586 * rint(a * 0.15915494309189535);
+    float sn, cs;
+    sincosf(static_cast<float>(r), &sn, &cs);
+    const float x = kx, y = ky;
+    kx = x * cs - y * sn;
+    ky = y * cs + x * sn;
   }
   p.k_out[row * kHeadDim + j] = __float2bfloat16_rn(kx);
   p.k_out[row * kHeadDim + j + 64] = __float2bfloat16_rn(ky);

@@ -71,6 +71,7 @@ def _check(pool, pool0, ref, rows, what):
     (64, 3, 8, 16, True, 16, 256, False),
     (130, 2, 4, 5, False, 0, 300, True),
     (33, 4, 8, 4, True, 64, 512, True),
+    (9, 5, 2, 2, False, 0, 40, True),       # 5 layers: K ranges not split (table of 16 entries)
 ])
 def test_projection_matches_oracle(T, L, hkv, C, paged, P, cap, rope):
     k_pool, v_pool, k0, v0, kref, vref, rows = _run_case(T, L, hkv, C, paged, P, cap, rope, seed=T + L + hkv)
