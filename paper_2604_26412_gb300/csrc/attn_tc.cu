@@ -5,28 +5,36 @@
 // tile (Sec. 2.2 Eq. "kv-reattention" over the memory M_i of Sec. 3.4 /
 // App. B, as an online softmax in the log2 domain):
 //   S = Q K^T      tcgen05.mma M=128 N=64  K=128 (8 x K16), A = Q (smem), B = K tile (smem), D = S (TMEM)
-//   P = softmax(S) one thread per row: TMEM -> registers -> bf16 P (smem, 128B-swizzled)
-//   O += P V       tcgen05.mma M=128 N=128 K=64 (4 x K16), A = P (smem), B = V tile (smem, MN-major), D = O (TMEM)
+//   P = softmax(S) TMEM -> registers -> bf16 pairs written back over the S columns (TMEM)
+//   O += P V       tcgen05.mma M=128 N=128 K=64 (4 x K16), A = P (TMEM), B = V tile (smem, MN-major), D = O (TMEM)
 // Warp roles: warps 0..7 are two softmax warpgroups; warps 10 and 9 load the
 // K and V tiles of even and odd tiles by TMA, warp 9 also the q blocks (a
 // single warp keeps too few bulk-tensor loads in flight to reach full HBM
-// bandwidth);
-// warp 11 owns TMEM and one of its threads issues every QK^T, one thread of
-// warp 8 every P.V.
-// Warpgroup w owns the tiles t with t % 2 == w: it turns S into P for all 64
-// keys with its own running max/sum and its own O accumulator O_w in TMEM, so
-// the two warpgroups' per-tile chains overlap; the states are merged by
-// log-sum-exp at the end of each piece.  S has four TMEM buffers; QK^T is
-// issued as soon as a K tile and an S buffer are free and P.V as soon as P is
-// written, so QK^T runs ahead of the softmax.  O_w is rescaled in
-// TMEM only when a row's running max grows by more than 2^8 (lazy rescale).
-// Rows of the 128-row MMA that hold no stacked row carry no output.
+// bandwidth); warp 11 owns TMEM and one of its threads issues every QK^T, one
+// thread of warp 8 every P.V.
+// Row modes (one kernel each):
+//  - dense (up to 128 rows, a thread per TMEM lane) and spread (up to 64 rows,
+//    16 per TMEM lane quarter, two threads per row): warpgroup w owns the tiles
+//    t with t % 2 == w, with its own running max/sum and its own O_w, so the
+//    two warpgroups' per-tile chains overlap; their states are merged by
+//    log-sum-exp at the end of each piece.  Four S buffers; an S buffer is
+//    free again when P.V of its tile completes.
+//  - paired (129..256 rows, attn_tc_pair_kernel): two 128-row blocks per unit,
+//    warpgroup w owning block w on every tile, so each K/V tile is read once
+//    for both.
+// O_w is rescaled in TMEM only when a row's running max grows by more than
+// 2^8 (lazy rescale).  Rows of the 128-row MMA that hold no stacked row carry
+// no output.
 // K and V tiles are staged in the grouped layout (kGroupBytes): one TMA box
 // brings a whole page of up to 64 tokens with both 64-dim halves, so a tile of
-// 16-token pages takes 4 boxes per tensor instead of 8.  Ring depths (4 K,
-// 5 V, 2 P buffers) were measured on GB300: the bytes in flight per SM that
-// the K and V rings allow bound how fast one CTA streams, and a third P buffer
-// gained nothing.
+// 16-token pages takes 4 boxes per tensor instead of 8.  Ring depths (5 K,
+// 6 V) were measured on GB300: the bytes in flight per SM that the rings
+// allow bound how fast one CTA streams.
+// fp8 target cache (dense and spread rows, when forced): the producer warps
+// land the e4m3 codes in slots of their own and decode them into f16 tiles;
+// q and the draft tiles are converted to f16 and the MMAs multiply in f16.
+#include <cuda_fp16.h>
+
 #include "kvshot_attn_common.cuh"
 #include "kvshot_tcgen05.cuh"
 
@@ -50,7 +58,13 @@ constexpr int kSoftmaxThreads = 256;       // two warpgroups
 constexpr int kBarSoftmax = 1;             // named barrier among the softmax warps
 constexpr uint32_t kTmemCols = 512;        // S0..S3 [0,256), O0 [256,384), O1 [384,512)
 constexpr uint32_t kTmemO = kNS * kTileKeys;
-constexpr int kMiscInts = 12;
+constexpr int kMiscInts = 20;
+// fp8 (e4m3) target cache: rings of bf16 tiles decoded by the producer warps, which land the codes in two
+// slots of their own (8 KB of K codes and 8 KB of V codes each).
+constexpr int kF8NK = 3;
+constexpr int kF8NV = 4;
+constexpr int kLandBytes = 2 * kTileKeys * 128;  // one landing slot: a tile's K codes then its V codes
+constexpr int kLandSlots = 2;                    // per producer warp: one own tile in flight, one decoding
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max grows by > 256x
 
 // Row modes.  Dense: one block of up to 128 stacked rows, one thread per TMEM lane, the two
@@ -64,6 +78,31 @@ struct RingOf {
   static constexpr int NK = M == kModePair ? kPairNK : kNK;
   static constexpr int NV = M == kModePair ? kPairNV : kNV;
 };
+
+__device__ __forceinline__ uint32_t pack_f16x2_tc(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void sts128(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
+// A buffer of bf16 values (whole 16-byte chunks, shared-memory address `buf`) converted in place to f16
+// by one warp: exact for magnitudes in [2^-14, 65504] (values below 2^-14 lose low bits).  The layout
+// (swizzle included) is kept, since every element stays where it was.
+__device__ __forceinline__ void bf16_to_f16_inplace(uint32_t buf, int bytes, int lane) {
+#pragma unroll 4
+  for (int off = lane * 16; off < bytes; off += 32 * 16) {
+    uint4 v = lds128(buf + off);
+    v.x = pack_f16x2_tc(bf16_lo(v.x), bf16_hi(v.x));
+    v.y = pack_f16x2_tc(bf16_lo(v.y), bf16_hi(v.y));
+    v.z = pack_f16x2_tc(bf16_lo(v.z), bf16_hi(v.z));
+    v.w = pack_f16x2_tc(bf16_lo(v.w), bf16_hi(v.w));
+    sts128(buf + off, v);
+  }
+}
 
 // Byte offset of 16-byte chunk `ch` (dims 8ch..8ch+7) of key r in a K or V
 // tile of either layout (128-byte swizzle: chunk index XOR row index mod 8).
@@ -79,6 +118,7 @@ struct Smem {
   uint8_t* kring;      // kNK x K tile
   uint8_t* vring;      // kNV x V tile
   uint8_t* qbuf;       // one q block
+  uint8_t* land;       // fp8 cache: [2 producer warps][kLandSlots] landing slots of e4m3 codes
   uint64_t* kfull;     // [kNK]  TMA -> MMA
   uint64_t* kempty;    // [kNK]  QK^T of the slot's tile completed -> TMA
   uint64_t* vfull;     // [kNV]  TMA -> MMA, softmax
@@ -91,19 +131,25 @@ struct Smem {
   uint64_t* pvdone;    // [kNW]  P.V into O_w of warpgroup w's latest tile completed
   uint64_t* ofree;     // [1]  epilogue finished reading O
   uint64_t* mmadone;   // [2]  every QK^T / every P.V completed
+  uint64_t* full8;     // fp8 cache: [2][kLandSlots] codes landed (TMA)
+  uint64_t* qland;     // fp8 cache: [1] bf16 q block landed (converted to f16 before qfull)
+  uint64_t* dland;     // fp8 cache: [2] a producer warp's bf16 draft tile landed (converted before kfull / vfull)
   uint64_t* anc;       // [64]
   int* par;            // [64]
   float* comb;         // [128][2] second warpgroup's (max, sum) per row at a piece end
   uint32_t* tmem_base;
   int* misc;           // [0] abort, [2] K tiles consumed, [3]/[4] q blocks issued/consumed, [6] V tiles consumed,
-                       // [8..9] / [10..11] K / V tiles issued per producer warp
+                       // [8..9] / [10..11] K / V tiles issued per producer warp, [12..13] / [14..15] fp8 landings
+                       // issued / decoded per producer warp, [1] fp8: q blocks converted, [16..17] / [18..19] fp8:
+                       // draft tiles landed / converted per producer warp
   int* len;
   int* base;
 };
 
-__host__ __device__ inline size_t smem_bytes(int C) {
-  size_t off = static_cast<size_t>(kNK + kNV) * kKVBytes + kQBufBytes;
-  off += sizeof(uint64_t) * (2 * kNK + 2 * kNV + 2 + 3 * kNS + kNW + 3);
+__host__ __device__ inline size_t smem_bytes(int C, bool f8) {
+  const int nk = f8 ? kF8NK : kNK, nv = f8 ? kF8NV : kNV;
+  size_t off = static_cast<size_t>(nk + nv) * kKVBytes + kQBufBytes + (f8 ? 2 * kLandSlots * kLandBytes : 0);
+  off += sizeof(uint64_t) * (2 * nk + 2 * nv + 2 + 3 * kNS + kNW + 3 + 2 * kLandSlots + 3);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(float) * 2 * kQRows;
   off += sizeof(uint32_t) * 4 + sizeof(int) * kMiscInts;
@@ -111,21 +157,24 @@ __host__ __device__ inline size_t smem_bytes(int C) {
   return off + 1024;
 }
 
-__device__ Smem carve(uint8_t* raw, int C) {
+__device__ Smem carve(uint8_t* raw, int C, bool f8) {
+  const int nk = f8 ? kF8NK : kNK, nv = f8 ? kF8NV : kNV;
   Smem s;
   uint8_t* p = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
   s.kring = p;
-  p += kNK * kKVBytes;
+  p += nk * kKVBytes;
   s.vring = p;
-  p += kNV * kKVBytes;
+  p += nv * kKVBytes;
   s.qbuf = p;
   p += kQBufBytes;
+  s.land = p;
+  if (f8) p += 2 * kLandSlots * kLandBytes;
   uint64_t* b = reinterpret_cast<uint64_t*>(p);
   s.kfull = b;
-  s.kempty = s.kfull + kNK;
-  s.vfull = s.kempty + kNK;
-  s.vempty = s.vfull + kNV;
-  s.qfull = s.vempty + kNV;
+  s.kempty = s.kfull + nk;
+  s.vfull = s.kempty + nk;
+  s.vempty = s.vfull + nv;
+  s.qfull = s.vempty + nv;
   s.qempty = s.qfull + 1;
   s.sfull = s.qempty + 1;
   s.sfree = s.sfull + kNS;
@@ -133,7 +182,10 @@ __device__ Smem carve(uint8_t* raw, int C) {
   s.pvdone = s.pfull + kNS;
   s.ofree = s.pvdone + kNW;
   s.mmadone = s.ofree + 1;
-  s.anc = s.mmadone + 2;
+  s.full8 = s.mmadone + 2;
+  s.qland = s.full8 + 2 * kLandSlots;
+  s.dland = s.qland + 1;
+  s.anc = s.dland + 2;
   s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
   s.comb = reinterpret_cast<float*>(s.par + kMaxTreeNodes);
   s.tmem_base = reinterpret_cast<uint32_t*>(s.comb + 2 * kQRows);
@@ -153,16 +205,19 @@ __device__ Smem carve(uint8_t* raw, int C) {
 // S = Q K^T of every tile.  Tile t needs its K tile, its S buffer freed by
 // the completion of P.V of tile t - kNS, and (first tile of a piece) the
 // piece's q block.
+template <bool kF8>
 __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                            Cursor cu) {
-  constexpr uint32_t idesc = idesc_bf16(128, 64, false);
+  // fp8 cache: q and the tiles are f16 (e4m3 -> f16 is one conversion per two codes).
+  constexpr uint32_t idesc = kF8 ? idesc_f16(128, 64, false) : idesc_bf16(128, 64, false);
+  constexpr int NK = kF8 ? kF8NK : kNK;
   int piece = 0;
   for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
     bool ok = !*pipe.abort;
     if (ok && ti.first) ok = mbar_wait(smem_addr(sm.qfull), piece & 1, p.err, p.wait_ns);
     if (ok && t >= kNS) ok = mbar_wait(smem_addr(&sm.sfree[t % kNS]), ((t - kNS) / kNS) & 1, p.err, p.wait_ns);
-    if (ok) ok = mbar_wait(smem_addr(&sm.kfull[t % kNK]), (t / kNK) & 1, p.err, p.wait_ns);
+    if (ok) ok = mbar_wait(smem_addr(&sm.kfull[t % NK]), (t / NK) & 1, p.err, p.wait_ns);
     if (!ok) {
       *pipe.abort = 1;
       break;
@@ -171,7 +226,7 @@ __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, 
     sm.misc[2] = t + 1;
     tc_fence_after();
     const uint32_t qbase = smem_addr(sm.qbuf);
-    const uint32_t kbase = smem_addr(sm.kring + static_cast<size_t>(t % kNK) * kKVBytes);
+    const uint32_t kbase = smem_addr(sm.kring + static_cast<size_t>(t % NK) * kKVBytes);
     // K tile: 8-key groups (the MMA's N direction) kGroupBytes apart and the dims 64..127 half
     // kGroupHalfBytes on (grouped layout), or 1 KB and kHalfBytes (halves layout).
     const bool grouped = ti.draft || p.prefix_grouped;
@@ -183,7 +238,7 @@ __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, 
       tc_mma(tmem + (t % kNS) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
     }
     tc_commit(smem_addr(&sm.sfull[t % kNS]));
-    tc_commit(smem_addr(&sm.kempty[t % kNK]));
+    tc_commit(smem_addr(&sm.kempty[t % NK]));
     if (ti.last) tc_commit(smem_addr(sm.qempty));
   }
   tc_commit(smem_addr(&sm.mmadone[0]));
@@ -194,9 +249,11 @@ __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, 
 // V tile; the first P.V into O_w of a piece (which overwrites O_w) needs the
 // previous piece's epilogue to have read O.  Each completion frees the tile's
 // S buffer for QK^T of tile t + kNS.
+template <bool kF8>
 __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                            Cursor cu) {
-  constexpr uint32_t idesc = idesc_bf16(128, 128, true);
+  constexpr uint32_t idesc = kF8 ? idesc_f16(128, 128, true) : idesc_bf16(128, 128, true);
+  constexpr int NV = kF8 ? kF8NV : kNV;
   int piece = 0, piece_t0 = 0;
   for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
@@ -208,7 +265,7 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
     bool ok = !*pipe.abort;
     if (ok && first && piece > 1) ok = mbar_wait(smem_addr(sm.ofree), (piece - 2) & 1, p.err, p.wait_ns);
     if (ok) ok = mbar_wait(smem_addr(&sm.pfull[t % kNS]), (t / kNS) & 1, p.err, p.wait_ns);
-    if (ok) ok = mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err, p.wait_ns);
+    if (ok) ok = mbar_wait(smem_addr(&sm.vfull[t % NV]), (t / NV) & 1, p.err, p.wait_ns);
     if (!ok) {
       *pipe.abort = 1;
       break;
@@ -216,7 +273,7 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
     sm.misc[6] = t + 1;
     tc_fence_after();
     const uint32_t pcol = tmem + (t % kNS) * kTileKeys;  // P: 32 columns of bf16 pairs
-    const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(t % kNV) * kKVBytes);
+    const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(t % NV) * kKVBytes);
     const uint32_t o = tmem + kTmemO + 128 * (t & 1);
     const bool grouped = ti.draft || p.prefix_grouped;
     const uint32_t half_off = grouped ? kGroupHalfBytes : kHalfBytes, group_off = grouped ? kGroupBytes : 1024;
@@ -226,7 +283,7 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
       const uint64_t bd = smem_desc_sw128(vbase + k16 * 2 * group_off, half_off, group_off);
       tc_mma_tmem_a(o, pcol + 8 * k16, bd, idesc, (first && k16 == 0) ? 0u : 1u);
     }
-    tc_commit(smem_addr(&sm.vempty[t % kNV]));
+    tc_commit(smem_addr(&sm.vempty[t % NV]));
     tc_commit(smem_addr(&sm.pvdone[t & 1]));
     tc_commit(smem_addr(&sm.sfree[t % kNS]));
   }
@@ -266,9 +323,10 @@ __device__ __forceinline__ void rescale_o_tmem(const Smem& sm, const Pipe& pipe,
   tmem_wait_st();
 }
 
-template <bool kSpread>
+template <bool kSpread, bool kF8>
 __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                             Cursor cu) {
+  constexpr int NV = kF8 ? kF8NV : kNV;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int quarter = warp & 3;                 // TMEM lanes this warp may access
   const int wg = warp >> 2;                     // warpgroup: owns tiles t with t % 2 == wg
@@ -357,19 +415,21 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
           }
         }
         const uint64_t vis = v64 >> col0;  // bit j = column col0 + j
+        // fp8 cache: the prefix keys' power-of-two scale is part of the score scale.
+        const float qs = (kF8 && !ti.draft) ? qscale * p.k_scale : qscale;
         float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
         // Dense rows skip the per-key mask on a full prefix tile (every key is visible): +6% on the
         // 128-row whole-tree stacks; spread rows (half the columns) measured ~2-4% slower with it.
         if (!kSpread && valid && !ti.draft && ti.nkeys >= kTileKeys) {
 #pragma unroll
           for (int j = 0; j < kCols; ++j) {
-            pr[j] = __uint_as_float(sv[j]) * qscale;
+            pr[j] = __uint_as_float(sv[j]) * qs;
             mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
           }
         } else {
 #pragma unroll
           for (int j = 0; j < kCols; ++j) {
-            pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * qscale : -INFINITY;
+            pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * qs : -INFINITY;
             mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
           }
         }
@@ -396,12 +456,14 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         const float m_use = m_run == -INFINITY ? 0.f : m_run;
         float ps4[4] = {0.f, 0.f, 0.f, 0.f};
         uint32_t pk[kCols / 2];  // P as bf16 pairs over the S columns just read (rows past the stack: zeros)
+        // fp8 cache: P of prefix tiles carries the values' power-of-two scale; the running sum does not.
+        const float vs = (kF8 && !ti.draft) ? p.v_scale : 1.f;
 #pragma unroll
         for (int j = 0; j < kCols / 2; ++j) {
           const float e0 = ex2(pr[2 * j] - m_use), e1 = ex2(pr[2 * j + 1] - m_use);
           ps4[(2 * j) & 3] += e0;
           ps4[(2 * j + 1) & 3] += e1;
-          pk[j] = pack_bf16x2(e0, e1);
+          pk[j] = kF8 ? pack_f16x2_tc(e0 * vs, e1 * vs) : pack_bf16x2(e0 * vs, e1 * vs);
         }
         l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
         if constexpr (kSpread) tmem_st16x2_16(trow + sbuf * kTileKeys, pk);
@@ -418,8 +480,8 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       if (live && warp_live) tmem_wait_st();
       if (live && ti.nkeys < kTileKeys) {
         // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.
-        if (!mbar_wait(smem_addr(&sm.vfull[t % kNV]), (t / kNV) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
-        uint8_t* vptr = sm.vring + static_cast<size_t>(t % kNV) * kKVBytes;
+        if (!mbar_wait(smem_addr(&sm.vfull[t % NV]), (t / NV) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
+        uint8_t* vptr = sm.vring + static_cast<size_t>(t % NV) * kKVBytes;
         const int nz = (kTileKeys - ti.nkeys) * 16;
         for (int i = wtid; i < nz; i += kSoftmaxThreads / 2) {
           const int key = ti.nkeys + (i >> 4), ch = i & 15;
@@ -722,6 +784,251 @@ __device__ __forceinline__ void run_producer_tc(const AttnParams& p, const Tenso
   }
 }
 
+
+
+// ------------------------------------------------------------ fp8 target cache
+
+// TMA boxes of the e4m3 codes of one prefix tile (2-D map {128 codes, rows}, boxes of whole 128-byte
+// rows, 128-byte swizzle): pages of P < 64 tokens one box each, larger pages and the contiguous cache
+// one 64-row box.  This lane's box is i = lane & 15; rows land in order at 128 bytes each.
+__device__ __forceinline__ TileBoxes tile_boxes_f8(const AttnParams& p, const Cursor& cu, PageWindow& win, int lane,
+                                                   int h, int pages, const FastDiv& pdiv) {
+  TileBoxes tb;
+  tb.draft = false;
+  tb.grouped = true;
+  tb.x = 0;
+  const int key0 = cu.lt * kTileKeys;
+  const int nkeys = min(kTileKeys, cu.L - key0);
+  const int i = lane & 15;
+  if (p.paged) {
+    const int P = p.page_size;
+    const bool small_pages = P < kTileKeys;
+    const int br = small_pages ? P : kTileKeys;
+    tb.nbox = small_pages ? pdiv.div(nkeys + P - 1) : 1;
+    const int pg0 = pdiv.div(key0);
+    win.cover(p, cu.c, pages, pg0, tb.nbox, lane);
+    const int pid = win.get(pg0 + (small_pages ? min(i, tb.nbox - 1) : 0));
+    tb.y = (pid * p.hkv + h) * P + (small_pages ? 0 : key0 - pg0 * P);
+    tb.off = static_cast<uint32_t>(i * br * 128);
+    tb.bytes = static_cast<uint32_t>(tb.nbox * br * 128);
+  } else {
+    tb.nbox = 1;
+    tb.y = (cu.c * p.hkv + h) * p.l_cap + key0;
+    tb.off = 0;
+    tb.bytes = kTileKeys * 128;
+  }
+  return tb;
+}
+
+// e4m3 codes of one landed K or V tile ([64 rows][128 codes], 128-byte swizzle) -> f16 in the grouped
+// layout, one hardware conversion per two codes (exact: 3 mantissa bits, exponents within f16's
+// normal range); the power-of-two scales are applied by the consumers.  Lane = one 16-code chunk of a
+// row per step (a warp reads 4 whole rows per step).
+__device__ __forceinline__ void decode_e4m3_tile(uint32_t src, uint32_t dst, int lane) {
+#pragma unroll 4
+  for (int it = 0; it < kTileKeys * 8 / 32; ++it) {
+    const int item = it * 32 + lane, r = item >> 3, c = item & 7;
+    const uint4 w = lds128(src + r * 128 + ((c ^ (r & 7)) << 4));
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+    uint32_t o[8];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %2;\n\t"
+          "cvt.rn.f16x2.e4m3x2 %0, lo;\n\tcvt.rn.f16x2.e4m3x2 %1, hi;\n\t}"
+          : "=r"(o[2 * k]), "=r"(o[2 * k + 1])
+          : "r"(ws[k]));
+    sts128(dst + tile_off_tc(r, 2 * c, true), make_uint4(o[0], o[1], o[2], o[3]));
+    sts128(dst + tile_off_tc(r, 2 * c + 1, true), make_uint4(o[4], o[5], o[6], o[7]));
+  }
+}
+
+// Producer warp `role` with an fp8 target cache.  For each of its tiles (t % 2 == role) it first lands
+// the codes of a prefix tile in its own slot (the n-th landing -> slot n % 2, one own tile ahead), then
+// finishes its oldest pending own tile: once that tile's K and V ring slots are free it decodes the landed
+// codes into them and arrives on kfull / vfull, or, for a draft tile (bf16), issues its loads straight
+// into the rings.  q blocks as in run_producer_tc (role 1).
+__device__ __forceinline__ void run_producer_f8(const AttnParams& p, const TensorMaps& maps, const Smem& sm,
+                                                const Pipe& pipe, Cursor cu, int nq_box, int role) {
+  constexpr int NK = kF8NK, NV = kF8NV;
+  const int lane = threadIdx.x & 31;
+  const uint64_t policy = l2_policy_evict_first();
+  PageWindow win;
+  int t = 0, piece = 0, landed = 0;  // landed: prefix tiles whose codes this warp has landed
+  const bool small = p.len_bound < (1 << 24) - 2 * kTileKeys;
+  const FastDiv pdiv(p.paged ? p.page_size : 1, small), rbdiv(p.row_blocks, true);
+  int unit_c = -1, unit_hr = -1, h = 0, pages = 0;
+  int ok = 1;
+  bool waited = false;
+  int drafts = 0, qblocks = 0;  // draft tiles this warp landed, q blocks it loaded
+  // Own tiles whose rings are not filled yet (oldest first, at most kLandSlots - 1): tile index,
+  // landing index (prefix tiles) and boxes.
+  constexpr int kPend = kLandSlots - 1;
+  int npend = 0, pend_t[kPend], pend_land[kPend];
+  TileBoxes pend_tb[kPend];
+  uint8_t* land = sm.land + static_cast<size_t>(role) * kLandSlots * kLandBytes;
+  // Fills the K and V ring slots of own tile x (boxes tb; a prefix tile's codes are landing jx).
+  auto finish = [&](int x, int jx, const TileBoxes& tb) -> bool {
+    const int kslot = x % NK, vslot = x % NV;
+    int good = 1;
+    if (lane < 2) {
+      const uint32_t bar = lane == 0 ? smem_addr(&sm.kempty[kslot]) : smem_addr(&sm.vempty[vslot]);
+      const uint32_t par = ((x / (lane == 0 ? NK : NV)) & 1) ^ 1u;
+      good = mbar_wait(bar, par, p.err, p.wait_ns) && !*pipe.abort;
+    }
+    if (!__all_sync(0xffffffffu, good)) return false;
+    uint8_t* kd = sm.kring + static_cast<size_t>(kslot) * kKVBytes;
+    uint8_t* vd = sm.vring + static_cast<size_t>(vslot) * kKVBytes;
+    if (tb.draft) {
+      if (!waited) {  // the draft K/V may come from the preceding kernel (KVSHOT_OVERLAP_PREVIOUS)
+        wait_for_prerequisite_grid();
+        waited = true;
+      }
+      // bf16 draft K/V land in the ring slots and are converted to f16 there.
+      const int kv = lane >> 4, i = lane & 15;
+      const uint32_t dbar = smem_addr(&sm.dland[role]);
+      if (lane == 0) mbar_arrive_expect_tx(dbar, 2 * tb.bytes);
+      __syncwarp();
+      if (i < tb.nbox) tma_load_3d(smem_addr(kv ? vd : kd) + tb.off, kv ? &maps.dv : &maps.dk, 0, tb.y, 0, dbar,
+                                   policy);
+      if (lane == 0) sm.misc[16 + role] = drafts + 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(dbar, drafts & 1, p.err, p.wait_ns))) return false;
+      ++drafts;
+      bf16_to_f16_inplace(smem_addr(kd), kKVBytes, lane);
+      bf16_to_f16_inplace(smem_addr(vd), kKVBytes, lane);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(smem_addr(&sm.kfull[kslot]));
+        mbar_arrive(smem_addr(&sm.vfull[vslot]));
+        sm.misc[18 + role] = drafts;
+      }
+    } else {
+      const int sl = jx % kLandSlots;
+      if (!mbar_wait(smem_addr(&sm.full8[role * kLandSlots + sl]), (jx / kLandSlots) & 1, p.err, p.wait_ns))
+        good = 0;
+      if (!__all_sync(0xffffffffu, good)) return false;
+      const uint32_t src = smem_addr(land + static_cast<size_t>(sl) * kLandBytes);
+      decode_e4m3_tile(src, smem_addr(kd), lane);
+      decode_e4m3_tile(src + kLandBytes / 2, smem_addr(vd), lane);
+      fence_proxy_async_smem();  // the MMAs read the tiles through the async proxy; the slot is reloaded by TMA
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(smem_addr(&sm.kfull[kslot]));
+        mbar_arrive(smem_addr(&sm.vfull[vslot]));
+        sm.misc[14 + role] = jx + 1;
+      }
+    }
+    if (lane == 0) {
+      sm.misc[8 + role] = x + 1;
+      sm.misc[10 + role] = x + 1;
+    }
+    return true;
+  };
+  for (; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
+    const bool first = cu.t == cu.t_begin || cu.lt == 0;  // first tile of a piece
+    const bool mine = (t & 1) == role;
+    if (!mine && !(first && role == 1)) {
+      piece += first;
+      continue;
+    }
+    if (cu.c != unit_c || cu.hr != unit_hr) {
+      unit_c = cu.c;
+      unit_hr = cu.hr;
+      h = rbdiv.div(cu.hr);
+      pages = p.paged ? pdiv.div(cu.L + p.page_size - 1) : 0;
+    }
+    if (first && role == 1) {  // the unit's q block
+      // The q buffer is released by QK^T of the previous piece's last tile, which may be this warp's
+      // pending tile: finish it before waiting.
+      bool good = true;
+      for (int k = 0; k < npend && good; ++k) good = finish(pend_t[k], pend_land[k], pend_tb[k]);
+      npend = 0;
+      if (!good) {
+        if (lane == 0) *pipe.abort = 1;
+        ok = 0;
+        break;
+      }
+      if (!waited) {
+        wait_for_prerequisite_grid();
+        waited = true;
+      }
+      if (lane == 0) {
+        const uint32_t qbar = smem_addr(sm.qland);  // converted to f16 below, then qfull
+        ok = mbar_wait(smem_addr(sm.qempty), (piece & 1) ^ 1u, p.err, p.wait_ns) && !*pipe.abort;
+        if (ok) {
+          const int rb = cu.hr - h * p.row_blocks;
+          const uint32_t dst = smem_addr(sm.qbuf);
+          const QBox qb = q_box(p.G, nq_box, nq_box * p.G <= kSpreadMaxRows);
+          const int box_rows = qb.heads * qb.nodes;
+          const int rows_q = p.G * nq_box;
+          const int nqb = nq_box * p.G <= kSpreadMaxRows ? (rows_q + box_rows - 1) / box_rows : 1;
+          mbar_arrive_expect_tx(qbar, 2 * nqb * box_rows * 128);
+          for (int k = 0; k < nqb; ++k) {
+            const int s0 = k * box_rows;
+            const uint32_t d = dst + k * 32 * 128;
+            tma_load_4d(d, &maps.q, 0, h * p.G + s0 % p.G, rb * nq_box + s0 / p.G, cu.c, qbar);
+            tma_load_4d(d + kQRows * 128, &maps.q, 64, h * p.G + s0 % p.G, rb * nq_box + s0 / p.G, cu.c, qbar);
+          }
+          sm.misc[3] = piece + 1;
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(smem_addr(sm.qland), qblocks & 1, p.err, p.wait_ns));
+      if (!ok) {
+        if (lane == 0) *pipe.abort = 1;
+        break;
+      }
+      ++qblocks;
+      bf16_to_f16_inplace(smem_addr(sm.qbuf), kQBufBytes, lane);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(smem_addr(sm.qfull));
+        sm.misc[1] = qblocks;
+      }
+    }
+    piece += first;
+    if (!mine) continue;
+    const bool draft = cu.lt >= cu.pt;
+    const TileBoxes tb = draft ? tile_boxes(p, cu, win, lane, h, pages, pdiv) : tile_boxes_f8(p, cu, win, lane, h,
+                                                                                                pages, pdiv);
+    if (!draft) {  // land the codes: landing n -> slot n % 2, free since landing n - 2 (an earlier tile) was decoded
+      const int sl = landed % kLandSlots;
+      const uint32_t fbar = smem_addr(&sm.full8[role * kLandSlots + sl]);
+      uint8_t* dst = land + static_cast<size_t>(sl) * kLandBytes;
+      const int kv = lane >> 4, i = lane & 15;
+      if ((lane & 15) == 0 && kv == 0) mbar_arrive_expect_tx(fbar, 2 * tb.bytes);
+      __syncwarp();
+      if (i < tb.nbox)
+        tma_load_2d(smem_addr(dst + kv * (kLandBytes / 2)) + tb.off, kv ? &maps.tv : &maps.tk, 0, tb.y, fbar, policy);
+      if (lane == 0) sm.misc[12 + role] = landed + 1;
+    }
+    if (npend == kPend) {  // the oldest pending tile, whose codes have had the longest to land
+      if (!finish(pend_t[0], pend_land[0], pend_tb[0])) {
+        ok = 0;
+        if (lane == 0) *pipe.abort = 1;
+        break;
+      }
+#pragma unroll
+      for (int k = 1; k < kPend; ++k) {
+        pend_t[k - 1] = pend_t[k];
+        pend_land[k - 1] = pend_land[k];
+        pend_tb[k - 1] = pend_tb[k];
+      }
+      --npend;
+    }
+    pend_t[npend] = t;
+    pend_land[npend] = landed;
+    pend_tb[npend] = tb;
+    ++npend;
+    landed += draft ? 0 : 1;
+  }
+  for (int k = 0; ok && k < npend; ++k)
+    if (!finish(pend_t[k], pend_land[k], pend_tb[k])) {
+      ok = 0;
+      if (lane == 0) *pipe.abort = 1;
+    }
+}
 
 // ============================================================ paired row blocks
 //
@@ -1169,15 +1476,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
 }
 
-template <bool kSpread>
+template <bool kSpread, bool kF8>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ TensorMaps maps, int nq_box) {
+  constexpr int NK = kF8 ? kF8NK : kNK, NV = kF8 ? kF8NV : kNV;
   extern __shared__ uint8_t smem_raw[];
   if (threadIdx.x == 0) allow_dependent_launch();  // the merge may be scheduled as CTAs finish
   // The plan's lengths are loaded first, so that their latency overlaps the set-up below
   // (a negative length, invalid anyway, is clamped by the ordinary path).
   const int len0 = static_cast<int>(threadIdx.x) < p.C ? p.seq_lens[threadIdx.x] : -1;
-  const Smem sm = carve(smem_raw, p.C);
+  const Smem sm = carve(smem_raw, p.C, kF8);
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 32 && p.paged) {
     // The page-table line of this CTA's first tile, were every length at its bound (exact
@@ -1192,11 +1500,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       asm volatile("prefetch.global.L2 [%0];" ::"l"(p.page_table + c * p.max_pages + pg));
   }
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kNK; ++s) {
+    for (int s = 0; s < NK; ++s) {
       mbar_init(smem_addr(&sm.kfull[s]), 1);
       mbar_init(smem_addr(&sm.kempty[s]), 1);
     }
-    for (int s = 0; s < kNV; ++s) {
+    for (int s = 0; s < NV; ++s) {
       mbar_init(smem_addr(&sm.vfull[s]), 1);
       mbar_init(smem_addr(&sm.vempty[s]), 1);
     }
@@ -1208,6 +1516,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads / 2);
     }
     for (int w = 0; w < kNW; ++w) mbar_init(smem_addr(&sm.pvdone[w]), 1);
+    if constexpr (kF8) {
+      for (int l = 0; l < 2 * kLandSlots; ++l) mbar_init(smem_addr(&sm.full8[l]), 1);
+      mbar_init(smem_addr(sm.qland), 1);
+      mbar_init(smem_addr(&sm.dland[0]), 1);
+      mbar_init(smem_addr(&sm.dland[1]), 1);
+    }
     mbar_init(smem_addr(sm.ofree), kSoftmaxThreads);
     mbar_init(smem_addr(&sm.mmadone[0]), 1);
     mbar_init(smem_addr(&sm.mmadone[1]), 1);
@@ -1230,12 +1544,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const Cursor cu = cursor_begin(p, sm.len, sm.base);
   Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), nullptr};
   if (warp == kProducerWarp || warp == kProducerVWarp) {
-    run_producer_tc<kSpread ? kModeSpread : kModeDense>(p, maps, sm, pipe, cu, nq_box, warp == kProducerWarp ? 0 : 1);
+    if constexpr (kF8) run_producer_f8(p, maps, sm, pipe, cu, nq_box, warp == kProducerWarp ? 0 : 1);
+    else run_producer_tc<kSpread ? kModeSpread : kModeDense>(p, maps, sm, pipe, cu, nq_box, warp == kProducerWarp ? 0 : 1);
   } else if (warp == kMmaWarp || warp == kMmaPvWarp) {
     const int stream = warp == kMmaWarp ? 0 : 1;
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
-      if (stream == 0) run_mma_qk(p, sm, pipe, tmem, cu);
-      else run_mma_pv(p, sm, pipe, tmem, cu);
+      if (stream == 0) run_mma_qk<kF8>(p, sm, pipe, tmem, cu);
+      else run_mma_pv<kF8>(p, sm, pipe, tmem, cu);
       // Every MMA must have completed before TMEM is released.  Each MMA issued reads shared memory
       // whose loads it already waited for, so it finishes; the wait is retried (bounded) if it runs
       // past its limit rather than freeing TMEM under a running MMA.
@@ -1244,7 +1559,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else if (warp < 8) {
-    run_softmax<kSpread>(p, sm, pipe, tmem, cu);
+    run_softmax<kSpread, kF8>(p, sm, pipe, tmem, cu);
   }
   tc_fence_before();
   __syncthreads();
@@ -1253,11 +1568,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     // A wait timed out: let every TMA load still in flight land before the CTA exits.
     // Tile k was loaded by producer warp k % 2, which issues its tiles in order.
     for (int k = sm.misc[2]; k < max(sm.misc[8], sm.misc[9]); ++k)
-      if (k < sm.misc[8 + (k & 1)] && !mbar_wait(smem_addr(&sm.kfull[k % kNK]), (k / kNK) & 1, p.err)) break;
+      if (k < sm.misc[8 + (k & 1)] && !mbar_wait(smem_addr(&sm.kfull[k % NK]), (k / NK) & 1, p.err)) break;
     for (int k = sm.misc[6]; k < max(sm.misc[10], sm.misc[11]); ++k)
-      if (k < sm.misc[10 + (k & 1)] && !mbar_wait(smem_addr(&sm.vfull[k % kNV]), (k / kNV) & 1, p.err)) break;
-    for (int k = sm.misc[4]; k < sm.misc[3]; ++k)
-      if (!mbar_wait(smem_addr(sm.qfull), k & 1, p.err)) break;
+      if (k < sm.misc[10 + (k & 1)] && !mbar_wait(smem_addr(&sm.vfull[k % NV]), (k / NV) & 1, p.err)) break;
+    if constexpr (!kF8) {
+      for (int k = sm.misc[4]; k < sm.misc[3]; ++k)
+        if (!mbar_wait(smem_addr(sm.qfull), k & 1, p.err)) break;
+    } else {
+      // q blocks, fp8 codes and draft tiles landed by the producer warps but not converted.
+      for (int k = sm.misc[1]; k < sm.misc[3]; ++k)
+        if (!mbar_wait(smem_addr(sm.qland), k & 1, p.err)) break;
+      for (int role = 0; role < 2; ++role) {
+        for (int j = sm.misc[14 + role]; j < sm.misc[12 + role]; ++j)
+          if (!mbar_wait(smem_addr(&sm.full8[role * kLandSlots + j % kLandSlots]), (j / kLandSlots) & 1, p.err))
+            break;
+        for (int j = sm.misc[18 + role]; j < sm.misc[16 + role]; ++j)
+          if (!mbar_wait(smem_addr(&sm.dland[role]), j & 1, p.err)) break;
+      }
+    }
   }
   if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
 }
@@ -1265,11 +1593,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 cudaError_t attn_tc_occupancy(int C, int* ctas_per_sm) {
-  const size_t smem = smem_bytes(C);
-  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  const size_t smem = smem_bytes(C, false);
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, attn_tc_kernel<false>, kThreads, smem);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, attn_tc_kernel<false, false>, kThreads, smem);
 }
 
 cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_box, bool spread, bool pair, bool pdl,
@@ -1282,8 +1610,10 @@ cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_b
     return launch_maybe_pdl(attn_tc_pair_kernel, dim3(p.num_ctas), dim3(kThreads), smem, pdl, stream, p, maps,
                             nq_box);
   }
-  const size_t smem = smem_bytes(p.C);
-  auto* kernel = spread ? attn_tc_kernel<true> : attn_tc_kernel<false>;
+  const bool f8 = p.fp8 != 0;
+  const size_t smem = smem_bytes(p.C, f8);
+  auto* kernel = f8 ? (spread ? attn_tc_kernel<true, true> : attn_tc_kernel<false, true>)
+                    : (spread ? attn_tc_kernel<true, false> : attn_tc_kernel<false, false>);
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   return launch_maybe_pdl(kernel, dim3(p.num_ctas), dim3(kThreads), smem, pdl, stream, p, maps, nq_box);

@@ -184,7 +184,10 @@ kvshot_status check_common(const kvshot_attn_desc* d) {
     if (d->k_scale_exp < -kMaxScaleExp || d->k_scale_exp > kMaxScaleExp || d->v_scale_exp < -kMaxScaleExp ||
         d->v_scale_exp > kMaxScaleExp)
       return KVSHOT_ERR_SHAPE;
-    if (d->flags & (KVSHOT_FORCE_CC | KVSHOT_FORCE_TC)) return KVSHOT_ERR_UNSUPPORTED;  // m16n8k16 kernel only
+    if (d->flags & KVSHOT_FORCE_CC) return KVSHOT_ERR_UNSUPPORTED;
+    // The tensor-memory kernel decodes fp8 tiles for stacks of up to 128 rows (not for paired blocks).
+    if ((d->flags & KVSHOT_FORCE_TC) && static_cast<int64_t>(d->hq / std::max(d->hkv, 1)) * d->n_query > 128)
+      return KVSHOT_ERR_UNSUPPORTED;
   }
   const uint32_t force = d->flags & (KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC);
   if (force & (force - 1)) return KVSHOT_ERR_SHAPE;  // at most one kernel may be forced
@@ -228,7 +231,10 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   //    shared memory into tensor memory, is faster (1.5x at 48 rows, 3-4x for
   //    whole-tree stacks of 128-256 rows).
   const bool tc_ok = G <= 128 && 128 % G == 0;
-  const bool fp8 = d->flags & KVSHOT_TARGET_FP8;  // only the m16n8k16 kernel decodes fp8 tiles
+  // fp8 tiles: both kernels decode them (the tensor-memory kernel only for stacks of up to 128 rows, when
+  // forced); decoding in registers (m16n8k16) measured faster on GB300 than decoding into shared memory for
+  // the tcgen05 MMAs (workload 3 per depth: 104 us against 112 us per call), so it is the default.
+  const bool fp8 = d->flags & KVSHOT_TARGET_FP8;
   const Kernel automatic = (rows > 16 && tc_ok && !fp8) ? Kernel::kTensorMemory : Kernel::kMma;
   pl->kernel = force_cc ? Kernel::kCudaCore : force_tc ? Kernel::kTensorMemory
                                            : force_mma ? Kernel::kMma : automatic;
@@ -349,7 +355,8 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   // The tensor-memory kernel stages tiles in the grouped layout: target tiles whenever their rows
   // start on a multiple of 8 (always when paged; contiguous caches with l_cap % 8 == 0), draft tiles always.
   const bool tmem_kernel = pl.kernel == Kernel::kTensorMemory;
-  const bool prefix_grouped = tmem_kernel && (paged || d->l_cap % 8 == 0);
+  // (fp8 prefix tiles are decoded into the grouped layout whatever the cache layout.)
+  const bool prefix_grouped = tmem_kernel && (fp8 || paged || d->l_cap % 8 == 0);
   bool tmaps;
   if (fp8) {
     tmaps = encode_rows_fp8(&maps.tk, target_k, trows, tbox) && encode_rows_fp8(&maps.tv, target_v, trows, tbox);

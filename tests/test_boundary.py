@@ -99,7 +99,9 @@ def _attn(d, **ptrs):
     (dict(flags=0x40), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=kvshot.KVSHOT_TARGET_FP8, k_scale_exp=65), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=kvshot.KVSHOT_TARGET_FP8, v_scale_exp=-65), kvshot.KVSHOT_ERR_SHAPE),
-    (dict(flags=kvshot.KVSHOT_TARGET_FP8 | kvshot.KVSHOT_FORCE_TC), kvshot.KVSHOT_ERR_UNSUPPORTED),
+    # fp8 on the tcgen05 kernel: stacks of up to 128 rows only (160 here: 40 query nodes x G = 4)
+    (dict(flags=kvshot.KVSHOT_TARGET_FP8 | kvshot.KVSHOT_FORCE_TC, n_nodes=40, n_query=40, n_max=40),
+     kvshot.KVSHOT_ERR_UNSUPPORTED),
     (dict(flags=kvshot.KVSHOT_TARGET_FP8 | kvshot.KVSHOT_FORCE_CC), kvshot.KVSHOT_ERR_UNSUPPORTED),
     (dict(flags=kvshot.KVSHOT_FORCE_CC | kvshot.KVSHOT_FORCE_MMA), kvshot.KVSHOT_ERR_SHAPE),
     (dict(flags=kvshot.KVSHOT_FORCE_MMA | kvshot.KVSHOT_FORCE_TC), kvshot.KVSHOT_ERR_SHAPE),

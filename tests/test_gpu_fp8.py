@@ -23,11 +23,13 @@ CASES = [
     ((0,), (1, 1, 1), False, False, 16, 32, 8, 1),                # empty prefix
     ((1, 63, 64, 65), (1, 1), False, True, 16, 32, 8, 1),         # ragged around the tile size
     ((17, 130, 300), (4, 4), True, True, 8, 32, 8, 4),            # tree, 16 rows, P = 8
-    ((4096, 1000), (8, 12, 12), True, True, 16, 32, 8, 12),       # 48 rows: m16n8k16 kernel (tcgen05 for bf16)
+    ((4096, 1000), (8, 12, 12), True, True, 16, 32, 8, 12),       # 48 rows (tcgen05 when forced: spread rows)
     ((257, 513), (8, 12, 12), True, True, 64, 32, 8, 32),         # 128 rows, row blocks
     ((700,), (2, 3, 3), True, True, 128, 32, 8, 8),               # page larger than a tile
     ((333, 5), (3, 3), True, False, 16, 8, 8, 3),                 # G = 1
     ((65,), tuple([1] * 70), False, False, 16, 4, 4, 2),          # chain with N = 70 > one draft tile
+    ((203, 64), tuple([1] * 40), False, False, 16, 32, 8, 32),    # 128 dense rows, contiguous l_cap % 8 != 0
+    ((300, 200), (8, 12, 12, 12), True, True, 16, 32, 8, 40),     # 160 rows: m16n8k16 only (no paired fp8 blocks)
 ]
 
 
@@ -70,10 +72,22 @@ def _run(spec, inp, tk8, tv8, dk, dv, q, N, Nq, flags, num_ctas=0):
 def test_fp8_target_matches_oracle(case):
     spec, inp, dk, dv, q, N, Nq, tk8, tv8, hc = _setup(case, seed=3 + len(case[0]) + sum(case[1]))
     ref_out, ref_lse = gh.oracle_attn(hc, q, dk, dv, N, Nq)
-    for flags in (0, kvshot.KVSHOT_FORCE_MMA):
+    rows = case[5] // case[6] * case[7]
+    for flags in (0, kvshot.KVSHOT_FORCE_MMA) + ((kvshot.KVSHOT_FORCE_TC,) if rows <= 128 else ()):
         for num_ctas in (0, 1, 7):
             out, lse = _run(spec, inp, tk8, tv8, dk, dv, q, N, Nq, flags, num_ctas)
             gh.compare(out, lse, ref_out, ref_lse, f"fp8 {case} flags={flags} ctas={num_ctas}")
+
+
+@pytest.mark.parametrize("nq", [12, 32])
+def test_fp8_tcgen05_matches_oracle_at_48_and_128_rows(nq):
+    # The tcgen05 kernel decoding fp8 tiles: 48 stacked rows (spread) and 128 (dense), paged P = 16.
+    case = ((3000, 517, 64), (8, 12, 12), True, True, 16, 32, 8, nq)
+    spec, inp, dk, dv, q, N, Nq, tk8, tv8, hc = _setup(case, seed=nq)
+    ref_out, ref_lse = gh.oracle_attn(hc, q, dk, dv, N, Nq)
+    for num_ctas in (0, 3, 152):
+        out, lse = _run(spec, inp, tk8, tv8, dk, dv, q, N, Nq, kvshot.KVSHOT_FORCE_TC, num_ctas)
+        gh.compare(out, lse, ref_out, ref_lse, f"fp8 tcgen05 nq={nq} ctas={num_ctas}")
 
 
 def test_fp8_is_deterministic_and_differs_from_bf16_only_by_quantisation():
