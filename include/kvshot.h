@@ -105,7 +105,7 @@ typedef struct kvshot_attn_desc {
   int32_t n_nodes;           /* N: draft nodes present; draft slots 0..N-1 hold their K/V */
   int32_t n_query;           /* Nq: the last Nq draft nodes are the query rows (Nq <= N) */
   int32_t n_max;             /* draft buffer capacity in slots (N <= n_max) */
-  float scale;               /* softmax scale on q.k; 0 selects 1/sqrt(head_dim) */
+  float scale;               /* softmax scale on q.k, > 0; 0 selects 1/sqrt(head_dim); negative -> KVSHOT_ERR_SHAPE */
   uint32_t flags;            /* KVSHOT_TREE, at most one of KVSHOT_FORCE_CC / _MMA / _TC */
   int32_t num_ctas;          /* persistent CTAs to launch; 0 = one full wave on this GPU */
   void* workspace;           /* device scratch, 256-byte aligned; see kvshot_draft_attn_workspace_size */
@@ -159,8 +159,9 @@ kvshot_status kvshot_draft_attn(const kvshot_attn_desc* desc, const void* q, con
                                 const void* draft_k, const void* draft_v, const int32_t* tree_parent,
                                 void* out, float* lse, kvshot_stream_t stream);
 
-/* Bytes of device scratch built into the library for kvshot_draft_attn_static (32 MiB). */
-#define KVSHOT_STATIC_WORKSPACE_BYTES (32u * 1024u * 1024u)
+/* Bytes of device scratch built into the library for kvshot_draft_attn_static (64 MiB: enough for the
+ * plan of a 64-node whole tree over 16 caches x 8 KV heads, 256 stacked rows per head, ~34 MB). */
+#define KVSHOT_STATIC_WORKSPACE_BYTES (64u * 1024u * 1024u)
 
 /*
  * kvshot_draft_attn_static -- the same computation, arguments and results as

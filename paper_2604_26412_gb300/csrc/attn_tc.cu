@@ -89,6 +89,58 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint4 v) {
                : "memory");
 }
 
+// Three-input maximum (one instruction on sm_100 and later).
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Two-lane fp32 FMA and add (one instruction each on sm_100 and later).
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+// Row maximum of N raw scores (four independent chains of three-input maxima).
+template <int N>
+__device__ __forceinline__ float row_max(const float (&s)[N]) {
+  float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+  for (int k = 0; k < N / 2; ++k) m4[k & 3] = max3(m4[k & 3], s[2 * k], s[2 * k + 1]);
+  return fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+}
+
+// P = 2^(s qs - m) of N raw scores (qs > 0), packed in pairs into pk (bf16, or f16 times vs), and the
+// sum of the unrounded values.  The scale rides in the exponent's FMA, two lanes per instruction.
+template <int N, bool kF16>
+__device__ __forceinline__ float row_exp(const float (&s)[N], float qs, float m, float vs, uint32_t (&pk)[N / 2]) {
+  const float2 q2 = make_float2(qs, qs), nm2 = make_float2(-m, -m);
+  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int k = 0; k < N / 2; ++k) {
+    const float2 x = fma2(make_float2(s[2 * k], s[2 * k + 1]), q2, nm2);
+    const float2 e = make_float2(ex2(x.x), ex2(x.y));
+    if (k & 1) acc1 = add2(acc1, e);
+    else acc0 = add2(acc0, e);
+    if constexpr (kF16) pk[k] = pack_f16x2_tc(e.x * vs, e.y * vs);
+    else pk[k] = pack_bf16x2(e.x, e.y);
+  }
+  return (acc0.x + acc0.y) + (acc1.x + acc1.y);
+}
+
 // A buffer of bf16 values (whole 16-byte chunks, shared-memory address `buf`) converted in place to f16
 // by one warp: exact for magnitudes in [2^-14, 65504] (values below 2^-14 lose low bits).  The layout
 // (swizzle included) is kept, since every element stays where it was.
@@ -418,22 +470,30 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         // fp8 cache: the prefix keys' power-of-two scale is part of the score scale.
         const float qs = (kF8 && !ti.draft) ? qscale * p.k_scale : qscale;
         float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        // Spread rows keep the raw scores and fold the scale into the exponent's argument,
+        // 2^(s qs - m) = ex2(fma(s, qs, -m)), with the row max taken on the raw scores (qs > 0), in
+        // two-lane FMAs and adds and three-input maxima (row_max, row_exp): fewer instructions per
+        // score (per-depth hybrid tree 55.0 -> 53.7 us per call on GB300 for the folded scale alone).
+        // Dense rows measured 2% slower with the folded scale and scale each score first.
+        const float pre = kSpread ? 1.f : qs;  // spread rows: pr holds the raw scores
         // Dense rows skip the per-key mask on a full prefix tile (every key is visible): +6% on the
         // 128-row whole-tree stacks; spread rows (half the columns) measured ~2-4% slower with it.
         if (!kSpread && valid && !ti.draft && ti.nkeys >= kTileKeys) {
 #pragma unroll
           for (int j = 0; j < kCols; ++j) {
-            pr[j] = __uint_as_float(sv[j]) * qs;
+            pr[j] = __uint_as_float(sv[j]) * pre;
             mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
           }
         } else {
 #pragma unroll
           for (int j = 0; j < kCols; ++j) {
-            pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * qs : -INFINITY;
-            mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
+            pr[j] = ((vis >> j) & 1u) ? __uint_as_float(sv[j]) * pre : -INFINITY;
+            if constexpr (!kSpread) mx4[j & 3] = fmaxf(mx4[j & 3], pr[j]);
           }
         }
-        float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+        float mx;
+        if constexpr (kSpread) mx = row_max(pr) * qs;
+        else mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
         if constexpr (kSpread) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
         // Lazy rescale: move this row's reference max only when it grows by > 2^8.  Dense rows rescale
         // O_wg after P is stored (below), so that P's 64 registers are free by then (it removed the
@@ -454,18 +514,22 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         }
         if (grow) m_run = mx;
         const float m_use = m_run == -INFINITY ? 0.f : m_run;
-        float ps4[4] = {0.f, 0.f, 0.f, 0.f};
         uint32_t pk[kCols / 2];  // P as bf16 pairs over the S columns just read (rows past the stack: zeros)
         // fp8 cache: P of prefix tiles carries the values' power-of-two scale; the running sum does not.
         const float vs = (kF8 && !ti.draft) ? p.v_scale : 1.f;
+        if constexpr (kSpread) {
+          l_run += row_exp<kCols, kF8>(pr, qs, m_use, vs, pk);
+        } else {
+          float ps4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int j = 0; j < kCols / 2; ++j) {
-          const float e0 = ex2(pr[2 * j] - m_use), e1 = ex2(pr[2 * j + 1] - m_use);
-          ps4[(2 * j) & 3] += e0;
-          ps4[(2 * j + 1) & 3] += e1;
-          pk[j] = kF8 ? pack_f16x2_tc(e0 * vs, e1 * vs) : pack_bf16x2(e0 * vs, e1 * vs);
+          for (int j = 0; j < kCols / 2; ++j) {
+            const float e0 = ex2(pr[2 * j] - m_use), e1 = ex2(pr[2 * j + 1] - m_use);
+            ps4[(2 * j) & 3] += e0;
+            ps4[(2 * j + 1) & 3] += e1;
+            pk[j] = kF8 ? pack_f16x2_tc(e0 * vs, e1 * vs) : pack_bf16x2(e0 * vs, e1 * vs);
+          }
+          l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
         }
-        l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
         if constexpr (kSpread) tmem_st16x2_16(trow + sbuf * kTileKeys, pk);
         else tmem_st32(trow + sbuf * kTileKeys, pk);
       }
@@ -1263,13 +1327,13 @@ __device__ __forceinline__ void run_softmax_pair(const AttnParams& p, const Smem
       tmem_ld32(my_s + j * kTileKeys, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
       tmem_ld32(my_s + j * kTileKeys + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
       tmem_wait_ld();
-      float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      // pr holds the raw scores; the scale is folded into the exponent's argument (row_exp),
+      // 2^(s qscale - m) = ex2(fma(s, qscale, -m)), and the row max is taken on the raw scores
+      // (qscale > 0; row_max): fewer instructions per score (whole-tree hybrid tree 99.4 -> 94.5 us
+      // per call for the folded scale alone).
       if (valid && !ti.draft && ti.nkeys >= kTileKeys) {  // a full prefix tile: every key is visible
 #pragma unroll
-        for (int k = 0; k < kTileKeys; ++k) {
-          pr[k] = __uint_as_float(sv[k]) * qscale;
-          mx4[k & 3] = fmaxf(mx4[k & 3], pr[k]);
-        }
+        for (int k = 0; k < kTileKeys; ++k) pr[k] = __uint_as_float(sv[k]);
       } else {
         uint64_t vis = 0;
         if (valid) {
@@ -1286,12 +1350,9 @@ __device__ __forceinline__ void run_softmax_pair(const AttnParams& p, const Smem
           }
         }
 #pragma unroll
-        for (int k = 0; k < kTileKeys; ++k) {
-          pr[k] = ((vis >> k) & 1u) ? __uint_as_float(sv[k]) * qscale : -INFINITY;
-          mx4[k & 3] = fmaxf(mx4[k & 3], pr[k]);
-        }
+        for (int k = 0; k < kTileKeys; ++k) pr[k] = ((vis >> k) & 1u) ? __uint_as_float(sv[k]) : -INFINITY;
       }
-      const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+      const float mx = row_max(pr) * qscale;
       // Lazy rescale: move this row's reference max only when it grows by > 2^8.
       const bool grow = valid && (m_run == -INFINITY ? mx != -INFINITY : mx > m_run + kRescaleThreshold);
       const bool rescale_o = grow && m_run != -INFINITY;
@@ -1300,16 +1361,8 @@ __device__ __forceinline__ void run_softmax_pair(const AttnParams& p, const Smem
       l_run *= alpha;
       if (grow) m_run = mx;
       const float m_use = m_run == -INFINITY ? 0.f : m_run;
-      float ps4[4] = {0.f, 0.f, 0.f, 0.f};
       uint32_t pk[kTileKeys / 2];  // P as bf16 pairs (rows past the stack hold zeros)
-#pragma unroll
-      for (int k = 0; k < kTileKeys / 2; ++k) {
-        const float e0 = ex2(pr[2 * k] - m_use), e1 = ex2(pr[2 * k + 1] - m_use);
-        ps4[(2 * k) & 3] += e0;
-        ps4[(2 * k + 1) & 3] += e1;
-        pk[k] = pack_bf16x2(e0, e1);
-      }
-      l_run += (ps4[0] + ps4[1]) + (ps4[2] + ps4[3]);
+      l_run += row_exp<kTileKeys, false>(pr, qscale, m_use, 1.f, pk);
       tmem_st32(my_s + j * kTileKeys, pk);  // P over the S columns just read
     }
     // P.V of the previous tile must complete before P of this tile is released: O_wg may then be

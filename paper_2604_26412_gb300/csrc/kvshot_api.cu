@@ -176,7 +176,7 @@ kvshot_status check_common(const kvshot_attn_desc* d) {
   if (d->head_dim != kHeadDim) return KVSHOT_ERR_UNSUPPORTED;
   if (d->n_nodes < 0 || d->n_query < 0 || d->n_query > d->n_nodes || d->n_nodes > d->n_max) return KVSHOT_ERR_SHAPE;
   if (d->max_seq_len < 0) return KVSHOT_ERR_SHAPE;
-  if (!std::isfinite(d->scale)) return KVSHOT_ERR_SHAPE;
+  if (!std::isfinite(d->scale) || d->scale < 0.f) return KVSHOT_ERR_SHAPE;  // the kernels fold a positive scale
   const uint32_t known =
       KVSHOT_TREE | KVSHOT_FORCE_CC | KVSHOT_FORCE_MMA | KVSHOT_FORCE_TC | KVSHOT_OVERLAP_PREVIOUS | KVSHOT_TARGET_FP8;
   if ((d->flags & ~known) != 0) return KVSHOT_ERR_SHAPE;

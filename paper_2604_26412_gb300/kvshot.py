@@ -38,7 +38,7 @@ EXPORTS = ("kvshot_draft_attn", "kvshot_draft_attn_workspace_size", "kvshot_draf
            "kvshot_version", "kvshot_draft_attn_static", "kvshot_gated_delta", "kvshot_gated_delta_workspace_size",
            "kvshot_kv_project", "kvshot_kv_project_workspace_size", "kvshot_draft_append_qknorm")
 KVSHOT_PROJECT_ROPE = 0x1
-STATIC_WORKSPACE_BYTES = 32 * 1024 * 1024  # KVSHOT_STATIC_WORKSPACE_BYTES
+STATIC_WORKSPACE_BYTES = 64 * 1024 * 1024  # KVSHOT_STATIC_WORKSPACE_BYTES
 
 
 class KvshotError(RuntimeError):

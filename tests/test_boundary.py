@@ -108,6 +108,7 @@ def _attn(d, **ptrs):
     (dict(flags=kvshot.KVSHOT_FORCE_TC, hq=24, hkv=8), kvshot.KVSHOT_ERR_UNSUPPORTED),
     (dict(num_ctas=-1), kvshot.KVSHOT_ERR_SHAPE),
     (dict(scale=float("inf")), kvshot.KVSHOT_ERR_SHAPE),
+    (dict(scale=-0.5), kvshot.KVSHOT_ERR_SHAPE),        # a softmax scale is positive (0 = default)
 ])
 def test_invalid_descriptor_codes(lib, kw, code):
     assert _attn(_desc(**kw)) == code
