@@ -21,7 +21,9 @@
 //    free again when P.V of its tile completes.
 //  - paired (129..256 rows, attn_tc_pair_kernel): two 128-row blocks per unit,
 //    warpgroup w owning block w on every tile, so each K/V tile is read once
-//    for both.
+//    for both.  14 warps: block 1 has QK^T and P.V issuers of its own (warps
+//    12, 13), so the two blocks' dependent MMA chains overlap in the tensor
+//    pipe and each block's commit waits for its own chain only.
 // O_w is rescaled in TMEM only when a row's running max grows by more than
 // 2^8 (lazy rescale).  Rows of the 128-row MMA that hold no stacked row carry
 // no output.
@@ -71,6 +73,9 @@ constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max
 // warpgroups alternating tiles.  Spread: up to 64 rows, 16 per TMEM lane quarter.  Pair: two
 // 128-row blocks of one KV head (129..256 rows), warpgroup w owning block w on every tile.
 constexpr int kModeDense = 0, kModeSpread = 1, kModePair = 2;
+constexpr int kPairThreads = 14 * 32;      // paired blocks: warps 12 and 13 issue QK^T and P.V of block 1
+constexpr int kMmaWarp1 = 12;              // paired blocks: QK^T issuer of block 1
+constexpr int kMmaPvWarp1 = 13;            // paired blocks: P.V issuer of block 1
 constexpr int kPairNK = 4;                 // paired blocks: K tiles in flight
 constexpr int kPairNV = 5;                 // paired blocks: V tiles in flight
 template <int M>
@@ -1112,9 +1117,9 @@ struct SmemPair {
   uint8_t* vring;      // kPairNV x V tile
   uint8_t* qbuf;       // Q_0, Q_1 (kQBufBytes each)
   uint64_t* kfull;     // [kPairNK]  TMA -> QK^T issuer
-  uint64_t* kempty;    // [kPairNK]  both QK^T of the tile completed -> TMA
+  uint64_t* kempty;    // [kPairNK]  both QK^T of the tile completed -> TMA (one commit per issuing thread)
   uint64_t* vfull;     // [kPairNV]  TMA -> P.V issuer (and warpgroup 0 on partial tiles)
-  uint64_t* vempty;    // [kPairNV]  both P.V of the tile completed -> TMA
+  uint64_t* vempty;    // [kPairNV]  both P.V of the tile completed -> TMA (one commit per issuing thread)
   uint64_t* qfull;     // [1]
   uint64_t* qempty;    // [1]
   uint64_t* sfull;     // [4]  S_{w,j} written (index 2 w + j)
@@ -1122,7 +1127,7 @@ struct SmemPair {
   uint64_t* pfull;     // [4]  P_w of a tile with parity j written over S_{w,j} (128 threads)
   uint64_t* pvdone;    // [2]  O_w += P_w V completed
   uint64_t* ofree;     // [2]  warpgroup w's epilogue read O_w (128 threads)
-  uint64_t* mmadone;   // [2]
+  uint64_t* mmadone;   // [4]  every MMA of an issuing thread completed (QK^T 0, 1, P.V 0, 1)
   uint64_t* anc;       // [64]
   int* par;            // [64]
   uint32_t* tmem_base;
@@ -1133,7 +1138,7 @@ struct SmemPair {
 
 __host__ __device__ inline size_t smem_bytes_pair(int C) {
   size_t off = static_cast<size_t>(kPairNK + kPairNV) * kKVBytes + 2 * kQBufBytes;
-  off += sizeof(uint64_t) * (2 * kPairNK + 2 * kPairNV + 2 + 4 + 4 + 4 + 2 + 2 + 2);
+  off += sizeof(uint64_t) * (2 * kPairNK + 2 * kPairNV + 2 + 4 + 4 + 4 + 2 + 2 + 4);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(uint32_t) * 4 + sizeof(int) * kMiscInts;
   off += sizeof(int) * (2 * C + 1);
@@ -1162,7 +1167,7 @@ __device__ SmemPair carve_pair(uint8_t* raw, int C) {
   s.pvdone = s.pfull + 4;
   s.ofree = s.pvdone + 2;
   s.mmadone = s.ofree + 2;
-  s.anc = s.mmadone + 2;
+  s.anc = s.mmadone + 4;
   s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
   s.tmem_base = reinterpret_cast<uint32_t*>(s.par + kMaxTreeNodes);
   s.misc = reinterpret_cast<int*>(s.tmem_base + 4);
@@ -1171,61 +1176,60 @@ __device__ SmemPair carve_pair(uint8_t* raw, int C) {
   return s;
 }
 
-// S_w = Q_w K^T of every tile for w = 0, 1.  Tile t needs its K tile, the
-// piece's q blocks (first tile of a piece) and, per block, S buffer (w, t & 1)
-// freed by the completion of P.V of tile t - 2.
+// S_w = Q_w K^T of every tile, for one block w (one issuing thread per block:
+// MMAs into one accumulator run one after another, each waiting for the last,
+// while those of the other block's thread overlap them; a commit tracks only
+// its own thread's MMAs, so S_w is released as soon as its own chain is done).
+// Tile t needs its K tile, the piece's q blocks (first tile of a piece) and S
+// buffer (w, t & 1), freed by the completion of P.V of block w of tile t - 2.
 __device__ __forceinline__ void run_mma_qk_pair(const AttnParams& p, const SmemPair& sm, const Pipe& pipe,
-                                                uint32_t tmem, Cursor cu) {
+                                                uint32_t tmem, Cursor cu, int w) {
   constexpr uint32_t idesc = idesc_bf16(128, 64, false);
   int piece = 0;
+  const uint32_t qbase = smem_addr(sm.qbuf + w * kQBufBytes);
   for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
     const int j = t & 1;
     bool ok = !*pipe.abort;
     if (ok && ti.first) ok = mbar_wait(smem_addr(sm.qfull), piece & 1, p.err, p.wait_ns);
     if (ok) ok = mbar_wait(smem_addr(&sm.kfull[t % kPairNK]), (t / kPairNK) & 1, p.err, p.wait_ns);
+    if (ok && t >= 2) ok = mbar_wait(smem_addr(&sm.sfree[2 * w + j]), ((t - 2) >> 1) & 1, p.err, p.wait_ns);
     if (!ok) {
       *pipe.abort = 1;
       break;
     }
-    if (ti.first) sm.misc[4] = ++piece;
-    sm.misc[2] = t + 1;
+    if (ti.first) ++piece;
+    if (w == 0) {
+      if (ti.first) sm.misc[4] = piece;
+      sm.misc[2] = t + 1;
+    }
+    tc_fence_after();
     const uint32_t kbase = smem_addr(sm.kring + static_cast<size_t>(t % kPairNK) * kKVBytes);
     const bool grouped = ti.draft || p.prefix_grouped;
     const uint32_t half_off = grouped ? kGroupHalfBytes : kHalfBytes, group_off = grouped ? kGroupBytes : 1024;
-    for (int w = 0; w < 2; ++w) {
-      if (t >= 2 && !mbar_wait(smem_addr(&sm.sfree[2 * w + j]), ((t - 2) >> 1) & 1, p.err, p.wait_ns)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      const uint32_t qbase = smem_addr(sm.qbuf + w * kQBufBytes);
 #pragma unroll
-      for (int ks = 0; ks < kHeadDim / 16; ++ks) {
-        const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
-        const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * half_off + (ks & 3) * 32, 16, group_off);
-        tc_mma(tmem + (2 * w + j) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
-      }
-      tc_commit(smem_addr(&sm.sfull[2 * w + j]));
+    for (int ks = 0; ks < kHeadDim / 16; ++ks) {
+      const uint64_t a = smem_desc_sw128(qbase + (ks >> 2) * (kQRows * 128) + (ks & 3) * 32, 16, 1024);
+      const uint64_t b = smem_desc_sw128(kbase + (ks >> 2) * half_off + (ks & 3) * 32, 16, group_off);
+      tc_mma(tmem + (2 * w + j) * kTileKeys, a, b, idesc, ks > 0 ? 1u : 0u);
     }
-    if (!ok) {
-      *pipe.abort = 1;
-      break;
-    }
-    tc_commit(smem_addr(&sm.kempty[t % kPairNK]));
-    if (ti.last) tc_commit(smem_addr(sm.qempty));
+    tc_commit(smem_addr(&sm.sfull[2 * w + j]));
+    tc_commit(smem_addr(&sm.kempty[t % kPairNK]));  // completes with both blocks' commits
+    if (ti.last) tc_commit(smem_addr(sm.qempty));   // likewise
   }
-  tc_commit(smem_addr(&sm.mmadone[0]));
+  tc_commit(smem_addr(&sm.mmadone[w]));
 }
 
-// O_w += P_w V of every tile for w = 0, 1, with P_w read from tensor memory
-// (the S columns of the tile).  The first P.V into O_w of a piece (which
-// overwrites O_w) needs the previous piece's epilogue to have read O_w.  Each
-// completion frees S buffer (w, t & 1) for QK^T of tile t + 2.
+// O_w += P_w V of every tile, for one block w (one issuing thread per block),
+// with P_w read from tensor memory (the S columns of the tile).  The first P.V
+// into O_w of a piece (which overwrites O_w) needs the previous piece's
+// epilogue to have read O_w.  Each completion frees S buffer (w, t & 1) for
+// QK^T of tile t + 2.
 __device__ __forceinline__ void run_mma_pv_pair(const AttnParams& p, const SmemPair& sm, const Pipe& pipe,
-                                                uint32_t tmem, Cursor cu) {
+                                                uint32_t tmem, Cursor cu, int w) {
   constexpr uint32_t idesc = idesc_bf16(128, 128, true);
   int piece = 0, piece_t0 = 0;
+  const uint32_t o = tmem + kTmemO + 128 * w;
   for (int t = 0; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
     const int j = t & 1;
@@ -1235,36 +1239,28 @@ __device__ __forceinline__ void run_mma_pv_pair(const AttnParams& p, const SmemP
     }
     bool ok = !*pipe.abort;
     if (ok) ok = mbar_wait(smem_addr(&sm.vfull[t % kPairNV]), (t / kPairNV) & 1, p.err, p.wait_ns);
+    if (ok && t == piece_t0 && piece > 1) ok = mbar_wait(smem_addr(&sm.ofree[w]), (piece - 2) & 1, p.err, p.wait_ns);
+    if (ok) ok = mbar_wait(smem_addr(&sm.pfull[2 * w + j]), (t >> 1) & 1, p.err, p.wait_ns);
     if (!ok) {
       *pipe.abort = 1;
       break;
     }
-    sm.misc[6] = t + 1;
+    if (w == 0) sm.misc[6] = t + 1;
+    tc_fence_after();
     const uint32_t vbase = smem_addr(sm.vring + static_cast<size_t>(t % kPairNV) * kKVBytes);
     const bool grouped = ti.draft || p.prefix_grouped;
     const uint32_t half_off = grouped ? kGroupHalfBytes : kHalfBytes, group_off = grouped ? kGroupBytes : 1024;
-    for (int w = 0; w < 2; ++w) {
-      if (t == piece_t0 && piece > 1) ok = mbar_wait(smem_addr(&sm.ofree[w]), (piece - 2) & 1, p.err, p.wait_ns);
-      if (ok) ok = mbar_wait(smem_addr(&sm.pfull[2 * w + j]), (t >> 1) & 1, p.err, p.wait_ns);
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t pcol = tmem + (2 * w + j) * kTileKeys;  // P_w: 32 columns of bf16 pairs
-      const uint32_t o = tmem + kTmemO + 128 * w;
+    const uint32_t pcol = tmem + (2 * w + j) * kTileKeys;  // P_w: 32 columns of bf16 pairs
 #pragma unroll
-      for (int k16 = 0; k16 < kTileKeys / 16; ++k16) {
-        const uint64_t bd = smem_desc_sw128(vbase + k16 * 2 * group_off, half_off, group_off);
-        tc_mma_tmem_a(o, pcol + 8 * k16, bd, idesc, (t == piece_t0 && k16 == 0) ? 0u : 1u);
-      }
-      tc_commit(smem_addr(&sm.pvdone[w]));
-      tc_commit(smem_addr(&sm.sfree[2 * w + j]));
+    for (int k16 = 0; k16 < kTileKeys / 16; ++k16) {
+      const uint64_t bd = smem_desc_sw128(vbase + k16 * 2 * group_off, half_off, group_off);
+      tc_mma_tmem_a(o, pcol + 8 * k16, bd, idesc, (t == piece_t0 && k16 == 0) ? 0u : 1u);
     }
-    if (!ok) {
-      *pipe.abort = 1;
-      break;
-    }
-    tc_commit(smem_addr(&sm.vempty[t % kPairNV]));
+    tc_commit(smem_addr(&sm.pvdone[w]));
+    tc_commit(smem_addr(&sm.sfree[2 * w + j]));
+    tc_commit(smem_addr(&sm.vempty[t % kPairNV]));  // completes with both blocks' commits
   }
-  tc_commit(smem_addr(&sm.mmadone[1]));
+  tc_commit(smem_addr(&sm.mmadone[2 + w]));
 }
 
 // Softmax and epilogue of warpgroup wg = block wg of every unit: thread =
@@ -1384,9 +1380,9 @@ __device__ __forceinline__ void run_softmax_pair(const AttnParams& p, const Smem
       }
       tmem_wait_st();
     }
-    if (wg == 0 && live && ti.nkeys < kTileKeys) {
-      // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.  Warpgroup 0 clears them
-      // before it releases P_0, and both P.V of the tile are issued after P_0's.
+    if (live && ti.nkeys < kTileKeys) {
+      // V rows past the valid keys may hold NaN; 0 * NaN would poison P.V.  Each warpgroup clears them
+      // before it releases its P (P.V of block w is issued after P_w alone; both write the same zeros).
       if (!mbar_wait(smem_addr(&sm.vfull[t % kPairNV]), (t / kPairNV) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
       uint8_t* vptr = sm.vring + static_cast<size_t>(t % kPairNV) * kKVBytes;
       const bool grouped = ti.draft || p.prefix_grouped;
@@ -1453,7 +1449,7 @@ __device__ __forceinline__ void run_softmax_pair(const AttnParams& p, const Smem
   }
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kPairThreads, 1)
     attn_tc_pair_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ TensorMaps maps, int nq_box) {
   extern __shared__ uint8_t smem_raw[];
   if (threadIdx.x == 0) allow_dependent_launch();  // the merge may be scheduled as CTAs finish
@@ -1463,23 +1459,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < kPairNK; ++s) {
       mbar_init(smem_addr(&sm.kfull[s]), 1);
-      mbar_init(smem_addr(&sm.kempty[s]), 1);
+      mbar_init(smem_addr(&sm.kempty[s]), 2);  // one commit per QK^T issuer
     }
     for (int s = 0; s < kPairNV; ++s) {
       mbar_init(smem_addr(&sm.vfull[s]), 1);
-      mbar_init(smem_addr(&sm.vempty[s]), 1);
+      mbar_init(smem_addr(&sm.vempty[s]), 2);  // one commit per P.V issuer
     }
     mbar_init(smem_addr(sm.qfull), 1);
-    mbar_init(smem_addr(sm.qempty), 1);
+    mbar_init(smem_addr(sm.qempty), 2);
     for (int b = 0; b < 4; ++b) {
       mbar_init(smem_addr(&sm.sfull[b]), 1);
       mbar_init(smem_addr(&sm.sfree[b]), 1);
       mbar_init(smem_addr(&sm.pfull[b]), kQRows);
+      mbar_init(smem_addr(&sm.mmadone[b]), 1);
     }
     for (int w = 0; w < 2; ++w) {
       mbar_init(smem_addr(&sm.pvdone[w]), 1);
       mbar_init(smem_addr(&sm.ofree[w]), kQRows);
-      mbar_init(smem_addr(&sm.mmadone[w]), 1);
     }
     for (int i = 0; i < kMiscInts; ++i) sm.misc[i] = 0;
     fence_mbar_init();
@@ -1501,13 +1497,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   Pipe pipe{nullptr, nullptr, nullptr, 0, reinterpret_cast<volatile int*>(&sm.misc[0]), nullptr};
   if (warp == kProducerWarp || warp == kProducerVWarp) {
     run_producer_tc<kModePair>(p, maps, sm, pipe, cu, nq_box, warp == kProducerWarp ? 0 : 1);
-  } else if (warp == kMmaWarp || warp == kMmaPvWarp) {
-    const int stream = warp == kMmaWarp ? 0 : 1;
+  } else if (warp == kMmaWarp || warp == kMmaPvWarp || warp == kMmaWarp1 || warp == kMmaPvWarp1) {
+    // One QK^T and one P.V issuer per block: warps 11, 8 for block 0 and 12, 13 for block 1.
+    const int w = (warp == kMmaWarp1 || warp == kMmaPvWarp1) ? 1 : 0;
+    const bool qk = warp == kMmaWarp || warp == kMmaWarp1;
     if ((threadIdx.x & 31) == 0 && cu.t < cu.t_end) {
-      if (stream == 0) run_mma_qk_pair(p, sm, pipe, tmem, cu);
-      else run_mma_pv_pair(p, sm, pipe, tmem, cu);
+      if (qk) run_mma_qk_pair(p, sm, pipe, tmem, cu, w);
+      else run_mma_pv_pair(p, sm, pipe, tmem, cu, w);
       // Every MMA must have completed before TMEM is released (retried, bounded, as in attn_tc_kernel).
-      for (int k = 0; k < 4 && !mbar_wait(smem_addr(&sm.mmadone[stream]), 0, p.err); ++k) {
+      const int done = qk ? w : 2 + w;
+      for (int k = 0; k < 4 && !mbar_wait(smem_addr(&sm.mmadone[done]), 0, p.err); ++k) {
       }
     }
     __syncwarp();
@@ -1660,7 +1659,7 @@ cudaError_t launch_attn_tc(const AttnParams& p, const TensorMaps& maps, int nq_b
     cudaError_t e = cudaFuncSetAttribute(attn_tc_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    return launch_maybe_pdl(attn_tc_pair_kernel, dim3(p.num_ctas), dim3(kThreads), smem, pdl, stream, p, maps,
+    return launch_maybe_pdl(attn_tc_pair_kernel, dim3(p.num_ctas), dim3(kPairThreads), smem, pdl, stream, p, maps,
                             nq_box);
   }
   const bool f8 = p.fp8 != 0;
