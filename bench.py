@@ -371,8 +371,16 @@ def call_roofline(step, inp, spec: wl.Spec, stream, ms_per_step: float, hbm_peak
     achieved_gbs = sum(call_bytes) / (sum(call_ms) / 1e3) / 1e9
     achieved_tflops = sum(call_flops) / (sum(call_ms) / 1e3) / 1e12
     G = spec.hq // spec.hkv
-    kernels = sorted({"tcgen05" if G * lv > 16 and 128 % G == 0 and target_elem == 2 else "m16n8k16"
-                      for lv in levels})
+    flags = step.descs[0].flags
+    if flags & kvshot.KVSHOT_FORCE_CC:
+        kernels = ["cuda-core"]
+    elif flags & kvshot.KVSHOT_FORCE_TC:
+        kernels = ["tcgen05"]
+    elif flags & kvshot.KVSHOT_FORCE_MMA:
+        kernels = ["m16n8k16"]
+    else:  # the library's automatic choice (kvshot_api.cu make_plan)
+        kernels = sorted({"tcgen05" if G * lv >= 16 and 128 % G == 0 and target_elem == 2 else "m16n8k16"
+                          for lv in levels})
     return {
         "bound": "hbm",
         "kernel": "kvshot_draft_attn (attention + merge kernels)",

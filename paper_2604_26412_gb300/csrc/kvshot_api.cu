@@ -222,20 +222,21 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   const bool force_cc = d->flags & KVSHOT_FORCE_CC, force_tc = d->flags & KVSHOT_FORCE_TC;
   const bool force_mma = d->flags & KVSHOT_FORCE_MMA;
   // Kernel choice, measured on GB300 (bench + ncu):
-  //  - up to 16 stacked rows per KV head the m16n8k16 kernel streams K/V at
-  //    90-98% of HBM bandwidth, also at 4 rows where the CUDA-core kernel is
-  //    issue bound (IPC ~1, ~100 warp instructions per key, 23%); the CUDA-core
+  //  - below 16 stacked rows per KV head the m16n8k16 kernel streams K/V at
+  //    90-94% of HBM bandwidth (4 rows: 187 us per ragged-chain call against
+  //    202 us for the tcgen05 kernel), also where the CUDA-core kernel is issue
+  //    bound (IPC ~1, ~100 warp instructions per key, 23%); the CUDA-core
   //    kernel stays behind KVSHOT_FORCE_CC;
-  //  - from 17 rows on, the mma.sync kernel becomes latency bound (one warp per
-  //    16-row tile) and the tcgen05 kernel, whose MMAs run asynchronously out of
-  //    shared memory into tensor memory, is faster (1.5x at 48 rows, 3-4x for
-  //    whole-tree stacks of 128-256 rows).
+  //  - from 16 rows on, the tcgen05 kernel, whose MMAs run asynchronously out
+  //    of shared memory into tensor memory, is faster: 314 us against 323 us
+  //    per multi-layer-tree call at 16 rows (spread rows), 1.9x at 48 rows,
+  //    3-4x for whole-tree stacks of 128-256 rows.
   const bool tc_ok = G <= 128 && 128 % G == 0;
   // fp8 tiles: both kernels decode them (the tensor-memory kernel only for stacks of up to 128 rows, when
   // forced); decoding in registers (m16n8k16) measured faster on GB300 than decoding into shared memory for
   // the tcgen05 MMAs (workload 3 per depth: 104 us against 112 us per call), so it is the default.
   const bool fp8 = d->flags & KVSHOT_TARGET_FP8;
-  const Kernel automatic = (rows > 16 && tc_ok && !fp8) ? Kernel::kTensorMemory : Kernel::kMma;
+  const Kernel automatic = (rows >= 16 && tc_ok && !fp8) ? Kernel::kTensorMemory : Kernel::kMma;
   pl->kernel = force_cc ? Kernel::kCudaCore : force_tc ? Kernel::kTensorMemory
                                            : force_mma ? Kernel::kMma : automatic;
   pl->mma = pl->kernel == Kernel::kMma;
