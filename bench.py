@@ -379,8 +379,10 @@ def call_roofline(step, inp, spec: wl.Spec, stream, ms_per_step: float, hbm_peak
     elif flags & kvshot.KVSHOT_FORCE_MMA:
         kernels = ["m16n8k16"]
     else:  # the library's automatic choice (kvshot_api.cu make_plan)
-        kernels = sorted({"tcgen05" if G * lv >= 16 and 128 % G == 0 and target_elem == 2 else "m16n8k16"
-                          for lv in levels})
+        def auto(rows):
+            tc = (16 < rows <= 128) if target_elem == 1 else rows >= 16
+            return "tcgen05" if tc and 128 % G == 0 else "m16n8k16"
+        kernels = sorted({auto(G * lv) for lv in levels})
     return {
         "bound": "hbm",
         "kernel": "kvshot_draft_attn (attention + merge kernels)",

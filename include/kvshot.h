@@ -76,11 +76,11 @@ typedef enum kvshot_status {
  * which is exact in bf16 for |exponent| <= 64; attention then proceeds as for a bf16 cache.  The
  * draft K/V stay bf16.  Both tensor-core kernels then multiply in f16 (e4m3 -> f16 is exact; q,
  * P and the draft K/V are rounded to f16, which keeps more mantissa than bf16; only magnitudes below
- * 2^-14 lose bits).  By default every stack runs on the m16n8k16 kernel, which decodes the codes in
- * registers; KVSHOT_FORCE_TC selects the tcgen05 kernel, which decodes them into f16 tiles in
- * shared memory, for stacks of up to 128 rows (more: KVSHOT_ERR_UNSUPPORTED).  KVSHOT_FORCE_CC
- * returns KVSHOT_ERR_UNSUPPORTED.  Not in the paper: a cache-compression variant that halves the
- * bytes the kernel reads per target token. */
+ * 2^-14 lose bits).  Stacks of 17 to 128 rows run on the tcgen05 kernel, which decodes the codes
+ * into f16 tiles in shared memory; the others on the m16n8k16 kernel, which decodes them in
+ * registers.  KVSHOT_FORCE_TC with more than 128 rows and KVSHOT_FORCE_CC return
+ * KVSHOT_ERR_UNSUPPORTED.  Not in the paper: a cache-compression variant that halves the bytes the
+ * kernel reads per target token. */
 #define KVSHOT_TARGET_FP8 0x20u
 
 /*

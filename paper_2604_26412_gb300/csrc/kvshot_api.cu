@@ -232,11 +232,13 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
   //    per multi-layer-tree call at 16 rows (spread rows), 1.9x at 48 rows,
   //    3-4x for whole-tree stacks of 128-256 rows.
   const bool tc_ok = G <= 128 && 128 % G == 0;
-  // fp8 tiles: both kernels decode them (the tensor-memory kernel only for stacks of up to 128 rows, when
-  // forced); decoding in registers (m16n8k16) measured faster on GB300 than decoding into shared memory for
-  // the tcgen05 MMAs (workload 3 per depth: 104 us against 112 us per call), so it is the default.
+  // fp8 tiles: both kernels decode them (the tensor-memory kernel for stacks of up to 128 rows).  The
+  // producer warps' decode into shared memory for the tcgen05 MMAs is the faster path for 17-128 rows
+  // (hybrid tree per depth, 32-48 rows: 85 us against 103 us per call for the m16n8k16 kernel, which
+  // decodes in registers); at 16 rows and below the m16n8k16 kernel is far ahead (264 us against 476 us).
   const bool fp8 = d->flags & KVSHOT_TARGET_FP8;
-  const Kernel automatic = (rows >= 16 && tc_ok && !fp8) ? Kernel::kTensorMemory : Kernel::kMma;
+  const bool tc_auto = fp8 ? (rows > 16 && rows <= 128) : rows >= 16;
+  const Kernel automatic = (tc_auto && tc_ok) ? Kernel::kTensorMemory : Kernel::kMma;
   pl->kernel = force_cc ? Kernel::kCudaCore : force_tc ? Kernel::kTensorMemory
                                            : force_mma ? Kernel::kMma : automatic;
   pl->mma = pl->kernel == Kernel::kMma;
