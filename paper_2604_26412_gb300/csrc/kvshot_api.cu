@@ -107,11 +107,12 @@ enum class Kernel { kCudaCore, kMma, kTensorMemory };
 // that stall the pipeline mid-stream, the merge kernel after the last CTA); measured on GB300.
 constexpr int64_t kSplitCostTiles = 15;
 
-// Fewest 64-key tiles per CTA of the m16n8k16 and CUDA-core kernels on an automatic grid: a CTA's
-// prologue and every extra piece to merge cost more than the parallelism of one-tile CTAs brings on
-// small, L2-resident problems (GB300: KV-only chain, 8 units of 33 tiles, 21.4 us per call on 264
-// CTAs against 14.4 us on 88; tiny chain, 8 units of 3 tiles, 11.8 against 10.5 us on 8 CTAs;
-// 2, 4, 6 or 8 tiles per CTA measured slower on both).  Large problems have hundreds of tiles per CTA.
+// Fewest 64-key tiles per CTA on an automatic grid: a CTA's prologue and every extra piece to merge
+// cost more than the parallelism of one-tile CTAs brings on small, L2-resident problems (GB300:
+// KV-only chain, 8 units of 33 tiles, m16n8k16 21.4 us per call on 264 CTAs against 14.4 us on 88,
+// tcgen05 whole chain 21.4 against 17.3 us on 88; tiny chain, 8 units of 3 tiles, 11.8 against
+// 10.5 us on 8 CTAs; 2, 4, 6 or 8 tiles per CTA measured slower).  Large problems have hundreds of
+// tiles per CTA.
 constexpr int64_t kMinTilesPerCta = 3;
 
 }  // namespace
@@ -296,7 +297,7 @@ kvshot_status make_plan(const kvshot_attn_desc* d, bool paged, Plan* pl) {
       if (unit_tiles * (grid - units) < kSplitCostTiles * static_cast<int64_t>(grid)) grid = static_cast<int>(units);
     }
   }
-  if (d->num_ctas == 0 && pl->kernel != Kernel::kTensorMemory)
+  if (d->num_ctas == 0)
     grid = static_cast<int>(std::min<int64_t>(grid, (max_tiles + kMinTilesPerCta - 1) / kMinTilesPerCta));
   grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(grid, std::max<int64_t>(1, max_tiles))));
   pl->num_ctas = grid;
