@@ -22,6 +22,11 @@
 // output columns are permuted too (n8 tile nd, column n -> dim 16 n + nd) and
 // the write-out undoes it.  Draft tiles (bf16) are read into the same layouts
 // and converted to f16 in registers.
+//
+// K/V tiles land in the halves layout (two 64-dim halves of 64 rows), or, for
+// a bf16 paged cache, in the grouped layout (8-row groups holding both halves):
+// there one TMA box brings a whole page of P < 64 tokens, or 8 draft slots,
+// which halves the boxes per tile (Cfg's GR flag).
 #include <cuda_fp16.h>
 
 #include "kvshot_attn_common.cuh"
@@ -83,9 +88,10 @@ __device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)
 constexpr int kBarConsumers = 1;
 constexpr int kCombStride = kHeadDim + 4;  // padded fp32 row in the combine buffer
 
-template <int MT, int KS, int STAGES, int MINB, bool F8 = false>
+template <int MT, int KS, int STAGES, int MINB, bool F8 = false, bool GR = false>
 struct Cfg {
   static constexpr bool kF8 = F8;                     // fp8 target tiles (KVSHOT_TARGET_FP8)
+  static constexpr bool kGrouped = GR;                // every tile in the grouped layout (bf16 paged caches)
   static constexpr int kMT = MT;                      // m16 tiles per unit
   static constexpr int kKS = KS;                      // key slices per tile
   static constexpr int kStages = STAGES;
@@ -338,6 +344,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
     const uint32_t kbase = smem_addr(kptr);
     const uint32_t vbase = kbase + kKVTileBytes;
     const bool f16t = CF::kF8 && !ti.draft;  // this tile's K/V are fp8 codes (scaled by 2^exp)
+    constexpr TileLayout lay = tile_layout(CF::kGrouped);
     if (!CF::kF8 && ti.nkeys < kTileKeys) {
       // V rows past the valid keys may be stale or NaN; the P.V product would
       // spread a NaN through 0 * NaN, so zero them (all consumer threads).  The
@@ -347,7 +354,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
         const int nz = (kTileKeys - ti.nkeys) * 16;  // 16-byte chunks to clear
         for (int i = threadIdx.x; i < nz; i += CF::kWarps * 32) {
           const int key = ti.nkeys + (i >> 4), ch = i & 15;
-          *reinterpret_cast<uint4*>(vptr + tile_off(key, ch)) = make_uint4(0, 0, 0, 0);
+          *reinterpret_cast<uint4*>(vptr + tile_off(key, ch, lay)) = make_uint4(0, 0, 0, 0);
         }
         fence_proxy_async_smem();
       }
@@ -380,7 +387,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
               b[0] = f0.x; b[1] = f0.y; b[2] = f1.x; b[3] = f1.y;
               b[4] = f2.x; b[5] = f2.y; b[6] = f3.x; b[7] = f3.y;
             } else {
-              const uint4 lo = lds128(kbase + tile_off(key, 2 * c)), hi = lds128(kbase + tile_off(key, 2 * c + 1));
+              const uint4 lo = lds128(kbase + tile_off(key, 2 * c, lay)), hi = lds128(kbase + tile_off(key, 2 * c + 1, lay));
               b[0] = bf16x2_to_f16x2(lo.x); b[1] = bf16x2_to_f16x2(lo.y);
               b[2] = bf16x2_to_f16x2(lo.z); b[3] = bf16x2_to_f16x2(lo.w);
               b[4] = bf16x2_to_f16x2(hi.x); b[5] = bf16x2_to_f16x2(hi.y);
@@ -399,7 +406,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
 #pragma unroll
           for (int kp = 0; kp < 4; ++kp) {
             uint32_t b0, b1, b2, b3;
-            ldmatrix_x4(kbase + tile_off(key, kp * 4 + lmat), b0, b1, b2, b3);
+            ldmatrix_x4(kbase + tile_off(key, kp * 4 + lmat, lay), b0, b1, b2, b3);
             mma_bf16_16816(s[j], qa[2 * kp], b0, b1);
             mma_bf16_16816(s[j], qa[2 * kp + 1], b2, b3);
           }
@@ -507,7 +514,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
               uint4 w[4];
 #pragma unroll
               for (int r = 0; r < 4; ++r) {
-                w[r] = lds128(vbase + tile_off(rows[r], 2 * g + hh));
+                w[r] = lds128(vbase + tile_off(rows[r], 2 * g + hh, lay));
                 if (rows[r] >= ti.nkeys) w[r] = make_uint4(0u, 0u, 0u, 0u);
               }
 #pragma unroll
@@ -525,7 +532,7 @@ __device__ __forceinline__ void run_consumer(const AttnParams& p, const Smem& sm
 #pragma unroll
           for (int ndp = 0; ndp < 8; ++ndp) {
             uint32_t b0, b1, b2, b3;
-            ldmatrix_x4_trans(vbase + tile_off(key, 2 * ndp + (lmat >> 1)), b0, b1, b2, b3);
+            ldmatrix_x4_trans(vbase + tile_off(key, 2 * ndp + (lmat >> 1), lay), b0, b1, b2, b3);
             mma_bf16_16816(o[2 * ndp], pa, b0, b1);
             mma_bf16_16816(o[2 * ndp + 1], pa, b2, b3);
           }
@@ -584,10 +591,10 @@ __global__ void __launch_bounds__(CF::kThreads, CF::kMinBlocks)
   if (threadIdx.x == 0) drain_after_abort(p, pipe, sm.misc[2]);
 }
 
-template <bool F8> using Cfg1 = Cfg<1, 4, 3, 2, F8>;
-template <bool F8> using Cfg2 = Cfg<2, 4, 4, 1, F8>;
-template <bool F8> using Cfg3 = Cfg<3, 2, 4, 1, F8>;
-template <bool F8> using Cfg4 = Cfg<4, 2, 4, 1, F8>;
+template <bool F8, bool GR = false> using Cfg1 = Cfg<1, 4, 3, 2, F8, GR>;
+template <bool F8, bool GR = false> using Cfg2 = Cfg<2, 4, 4, 1, F8, GR>;
+template <bool F8, bool GR = false> using Cfg3 = Cfg<3, 2, 4, 1, F8, GR>;
+template <bool F8, bool GR = false> using Cfg4 = Cfg<4, 2, 4, 1, F8, GR>;
 
 template <class CF>
 cudaError_t launch_cfg(const AttnParams& p, const TensorMaps& maps, bool pdl, cudaStream_t stream) {
@@ -626,19 +633,24 @@ cudaError_t attn_mma_occupancy(int m_tiles, int C, bool fp8, int* ctas_per_sm) {
   return fp8 ? occupancy_f8<true>(m_tiles, C, ctas_per_sm) : occupancy_f8<false>(m_tiles, C, ctas_per_sm);
 }
 
-template <bool F8>
+template <bool F8, bool GR>
 cudaError_t launch_f8(const AttnParams& p, const TensorMaps& maps, int m_tiles, bool pdl, cudaStream_t stream) {
   switch (m_tiles) {
-    case 1: return launch_cfg<Cfg1<F8>>(p, maps, pdl, stream);
-    case 2: return launch_cfg<Cfg2<F8>>(p, maps, pdl, stream);
-    case 3: return launch_cfg<Cfg3<F8>>(p, maps, pdl, stream);
-    case 4: return launch_cfg<Cfg4<F8>>(p, maps, pdl, stream);
+    case 1: return launch_cfg<Cfg1<F8, GR>>(p, maps, pdl, stream);
+    case 2: return launch_cfg<Cfg2<F8, GR>>(p, maps, pdl, stream);
+    case 3: return launch_cfg<Cfg3<F8, GR>>(p, maps, pdl, stream);
+    case 4: return launch_cfg<Cfg4<F8, GR>>(p, maps, pdl, stream);
     default: return cudaErrorInvalidValue;
   }
 }
 
+// The grouped instantiations (p.prefix_grouped: bf16 paged caches) have the resources of the
+// halves ones (same shared memory, registers capped by the same launch bounds), so the occupancy
+// query above serves both.
 cudaError_t launch_attn_mma(const AttnParams& p, const TensorMaps& maps, int m_tiles, bool pdl, cudaStream_t stream) {
-  return p.fp8 ? launch_f8<true>(p, maps, m_tiles, pdl, stream) : launch_f8<false>(p, maps, m_tiles, pdl, stream);
+  if (p.fp8) return launch_f8<true, false>(p, maps, m_tiles, pdl, stream);
+  return p.prefix_grouped ? launch_f8<false, true>(p, maps, m_tiles, pdl, stream)
+                          : launch_f8<false, false>(p, maps, m_tiles, pdl, stream);
 }
 
 }  // namespace kvshot

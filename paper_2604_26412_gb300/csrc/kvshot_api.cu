@@ -368,8 +368,13 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   // The tensor-memory kernel stages tiles in the grouped layout: target tiles whenever their rows
   // start on a multiple of 8 (always when paged; contiguous caches with l_cap % 8 == 0), draft tiles always.
   const bool tmem_kernel = pl.kernel == Kernel::kTensorMemory;
-  // (fp8 prefix tiles are decoded into the grouped layout whatever the cache layout.)
-  const bool prefix_grouped = tmem_kernel && (fp8 || paged || d->l_cap % 8 == 0);
+  // (fp8 prefix tiles are decoded into the grouped layout whatever the cache layout.)  The m16n8k16
+  // kernel stages every tile of a bf16 paged cache grouped too (prefix_grouped then covers its draft
+  // tiles): one box per page with both halves halves the TMA boxes a tile takes, which bounds small
+  // pages (GB300, ragged chain of 64 caches: 8-token pages 0.75 -> 0.92 of the copy peak, 16-token
+  // pages 0.93 -> 0.94).
+  const bool prefix_grouped =
+      tmem_kernel ? (fp8 || paged || d->l_cap % 8 == 0) : (pl.kernel == Kernel::kMma && paged && !fp8);
   bool tmaps;
   if (fp8) {
     tmaps = encode_rows_fp8(&maps.tk, target_k, trows, tbox) && encode_rows_fp8(&maps.tv, target_v, trows, tbox);
@@ -380,7 +385,7 @@ extern "C" kvshot_status kvshot_draft_attn(const kvshot_attn_desc* d, const void
   } else {
     tmaps = encode_rows(&maps.tk, target_k, trows, tbox) && encode_rows(&maps.tv, target_v, trows, tbox);
   }
-  const bool dmaps = tmem_kernel ? encode_rows_group3(&maps.dk, draft_k, drows) &&
+  const bool dmaps = tmem_kernel || prefix_grouped ? encode_rows_group3(&maps.dk, draft_k, drows) &&
                                        encode_rows_group3(&maps.dv, draft_v, drows)
                                  : encode_rows(&maps.dk, draft_k, drows, kDraftBoxRows) &&
                                        encode_rows(&maps.dv, draft_v, drows, kDraftBoxRows);

@@ -232,6 +232,22 @@ __device__ __forceinline__ uint32_t tile_off(int r, int ch) {
   return static_cast<uint32_t>((ch >> 3) * kHalfBytes + r * 128 + (((ch & 7) ^ (r & 7)) << 4));
 }
 
+// The same offset for a tile in either layout, given the strides of its 8-row
+// groups and of its 64-dim halves: {1024, kHalfBytes} for the halves layout
+// above, {kGroupBytes, kGroupHalfBytes} for the grouped layout (8-row groups of
+// both halves, as a grouped box lands).  The swizzle is the same in both.
+struct TileLayout {
+  uint32_t group, half;
+};
+__host__ __device__ constexpr TileLayout tile_layout(bool grouped) {
+  return grouped ? TileLayout{kGroupBytes, kGroupHalfBytes} : TileLayout{1024u, static_cast<uint32_t>(kHalfBytes)};
+}
+__device__ __forceinline__ uint32_t tile_off(int r, int ch, TileLayout l) {
+  if (l.group == 1024u && l.half == static_cast<uint32_t>(kHalfBytes)) return tile_off(r, ch);
+  return static_cast<uint32_t>(r >> 3) * l.group + static_cast<uint32_t>(ch >> 3) * l.half +
+         static_cast<uint32_t>(((r & 7) << 7) + (((ch & 7) ^ (r & 7)) << 4));
+}
+
 // ------------------------------------------------------------ work plan
 
 // Clamped prefix length of cache c; out-of-range values are reported.
@@ -531,13 +547,43 @@ __device__ __forceinline__ void run_producer(const AttnParams& p, const TensorMa
       const uint32_t kdst = smem_addr(pipe.ring + static_cast<size_t>(stage) * kStageBytes);
       const int kv = lane & 1, hf = (lane >> 1) & 1, i = lane >> 2;
       const uint32_t dst = kdst + kv * kKVTileBytes + hf * kHalfBytes;
-      if (draft) {
+      if (draft && p.prefix_grouped) {
+        // Grouped layout: box = lane -> (tensor K/V = lane & 1, 8-slot group lane >> 1), both halves
+        // (3-D map {64 dims, rows, 2 halves}).
+        const int nbox = (nkeys + kDraftBoxRows - 1) / kDraftBoxRows;
+        if (lane == 0) mbar_arrive_expect_tx(full_bar, 2u * nbox * kGroupBytes);
+        const int ib = lane >> 1;
+        if (ib < nbox) {
+          const int y0 = (cu.c * p.hkv + h) * p.n_max + key0;
+          tma_load_3d(kdst + kv * kKVTileBytes + ib * kGroupBytes, kv ? &maps.dv : &maps.dk, 0,
+                      y0 + ib * kDraftBoxRows, 0, full_bar, policy);
+        }
+      } else if (draft) {
         const int nbox = (nkeys + kDraftBoxRows - 1) / kDraftBoxRows;
         if (lane == 0) mbar_arrive_expect_tx(full_bar, nbox * kDraftBoxRows * 128 * 4);
         if (i < nbox) {
           const int y0 = (cu.c * p.hkv + h) * p.n_max + key0;
           tma_load_2d(dst + i * kDraftBoxRows * 128, kv ? &maps.dv : &maps.dk, hf * 64, y0 + i * kDraftBoxRows,
                       full_bar, policy);
+        }
+      } else if (p.paged && p.prefix_grouped) {
+        // Grouped layout (bf16): box = lane -> (tensor K/V = lane & 1, box lane >> 1), a box of whole
+        // 8-key groups with both 64-dim halves: one page of P < 64 tokens, or the tile's 64-token
+        // slice of a larger page.  Half the boxes of the halves layout, each twice the bytes.
+        const int P = p.page_size;
+        const bool small_pages = P < kTileKeys;
+        const int nbox = small_pages ? (nkeys + P - 1) / P : 1;
+        const uint32_t box_bytes = small_pages ? static_cast<uint32_t>(P) * 256u : static_cast<uint32_t>(kKVTileBytes);
+        if (lane == 0) mbar_arrive_expect_tx(full_bar, 2u * nbox * box_bytes);
+        const int ib = lane >> 1;
+        if (ib < nbox) {
+          int pid = pids[0];
+#pragma unroll
+          for (int k = 1; k < kTileKeys / 8; ++k)
+            if (ib == k) pid = pids[k];
+          const int y = ((pid * p.hkv + h) * P + (small_pages ? 0 : key0 % P)) >> 3;
+          tma_load_4d_hint(kdst + kv * kKVTileBytes + ib * box_bytes, kv ? &maps.tv : &maps.tk, 0, 0, 0, y,
+                           full_bar, policy);
         }
       } else if (p.paged) {
         // bf16: boxes of 64 dims per half; fp8 (p.fp8): one box of whole 128-byte rows, into the

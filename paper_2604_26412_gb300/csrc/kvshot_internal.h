@@ -77,7 +77,8 @@ struct AttnParams {
   float qscale;             // softmax scale * log2(e): scores are kept in the log2 domain
   int num_ctas;             // persistent grid size
   int fp8;                  // target K/V are e4m3 codes (KVSHOT_TARGET_FP8; m16n8k16 kernel only)
-  int prefix_grouped;       // tensor-memory kernel: prefix tiles are staged in the grouped layout (draft tiles always)
+  int prefix_grouped;       // prefix tiles are staged in the grouped layout (tensor-memory kernel: draft tiles always;
+                            // m16n8k16 kernel: draft tiles too)
   uint32_t wait_ns;         // limit on any one pipeline wait (desc->wait_limit_ns, default 2 s)
   float k_scale, v_scale;   // fp8: 2^k_scale_exp, 2^v_scale_exp
 };

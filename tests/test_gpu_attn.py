@@ -77,6 +77,8 @@ CASES = [
     ((203,), tuple([1] * 40), False, False, 16, 32, 8, 40),       # whole chain: paired, contiguous l_cap % 8 != 0
     ((96, 200), tuple([1] * 100), False, True, 16, 32, 8, 100),   # 400 rows: two paired units per KV head
     ((500,), (4, 8, 8), True, True, 64, 64, 8, 20),               # G = 8: 160 rows paired, 64-token pages
+    ((450, 31, 97), (2, 2), True, True, 32, 32, 8, 2),            # 32-token pages, ragged last page
+    ((700, 65), (1, 1, 1), False, True, 192, 32, 8, 1),           # 192-token pages: 64-token slices of a page
 ]
 
 
