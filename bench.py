@@ -145,10 +145,11 @@ def kernel_source_hash(sources=ATTN_SOURCES):
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload, mode, sources=ATTN_SOURCES):
+def recorded_traffic(workload, mode, sources=ATTN_SOURCES, kernel=None):
     """DRAM bytes per call (key "w<workload>-<mode>", or "fusion-hybrid_tree") from a committed ncu
-    summary, if it is for the current kernel sources; else None.  The record's "sources" (default:
-    `sources`) are the files its "kernel_hash" covers."""
+    summary, if it is for the current kernel sources (and, given `kernel`, for the attention kernel
+    that ran: the record's "kernel"); else None.  The record's "sources" (default: `sources`) are the
+    files its "kernel_hash" covers."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
@@ -158,6 +159,8 @@ def recorded_traffic(workload, mode, sources=ATTN_SOURCES):
     key = f"w{workload}-{mode}" if workload is not None else mode
     e = rec.get(key)
     if not e or e.get("kernel_hash") != kernel_source_hash(tuple(e.get("sources", sources))):
+        return None
+    if kernel is not None and e.get("kernel") != kernel:
         return None
     return e.get("dram_bytes_per_call")
 
@@ -341,11 +344,13 @@ def roofline_bytes(spec: wl.Spec, levels, paged: bool, fp8: bool):
     return [algorithmic_bytes(spec, n0s[i] + levels[i], levels[i], paged, 1 if fp8 else 2) for i in range(len(levels))]
 
 
-def call_roofline(step, inp, spec: wl.Spec, stream, ms_per_step: float, hbm_peak: float, peak_src: str, traffic=None,
-                  target_elem: int = 2) -> dict:
+def call_roofline(step, inp, spec: wl.Spec, stream, ms_per_step: float, hbm_peak: float, peak_src: str,
+                  traffic_key=None, target_elem: int = 2) -> dict:
     """Live roofline of the draft-attention calls of one step (attention + merge kernels): CUDA events
     around every call on the launching stream, the stream kept busy by a sleep kernel while the host
-    enqueues them; achieved = algorithmic bytes / mean call time."""
+    enqueues them; achieved = algorithmic bytes / mean call time.  traffic_key: (workload, mode) of
+    the committed traffic record for this exact configuration, or None; the record is used only if
+    one attention kernel ran and it is the record's."""
     from paper_2604_26412_gb300 import kvshot
     levels = step.levels
     n0s = np.cumsum([0] + levels[:-1]).tolist()
@@ -383,6 +388,9 @@ def call_roofline(step, inp, spec: wl.Spec, stream, ms_per_step: float, hbm_peak
             tc = (16 < rows <= 128) if target_elem == 1 else rows >= 16
             return "tcgen05" if tc and 128 % G == 0 else "m16n8k16"
         kernels = sorted({auto(G * lv) for lv in levels})
+    traffic = None
+    if traffic_key is not None and len(kernels) == 1:
+        traffic = recorded_traffic(*traffic_key, kernel=kernels[0])
     return {
         "bound": "hbm",
         "kernel": "kvshot_draft_attn (attention + merge kernels)",
@@ -423,7 +431,7 @@ def gate_roofline(workload: int, args, dev, hbm_peak: float, peak_src: str) -> d
         s1.record(stream)
     torch.cuda.synchronize()
     r = call_roofline(step, inp, spec, stream, s0.elapsed_time(s1) / 5, hbm_peak, peak_src,
-                      traffic=recorded_traffic(workload, "per_depth"))
+                      traffic_key=(workload, "per_depth"))
     out = {"workload": spec.name, "mode": "per_depth"}
     out.update({k: r[k] for k in ("frac", "achieved", "unit", "call_us", "per_level_us", "traffic",
                                   "algorithmic_bytes_per_call", "attention_kernels", "calls_timed")})
@@ -502,8 +510,10 @@ def run_ours(args, world, rank, local):
     # ---- live roofline of the draft-attention call (attention + merge kernels), per level
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    # A traffic record holds for the stock workload only (no prefix cap, page size or grid override).
+    stock = not args.max_prefix and not args.page_size and not args.num_ctas
     roofline = call_roofline(step, inp, spec, stream, ms_per_step, hbm_peak, peak_src,
-                             traffic=recorded_traffic(args.workload, args.mode + ("-fp8" if fp8 else "")),
+                             traffic_key=(args.workload, args.mode + ("-fp8" if fp8 else "")) if stock else None,
                              target_elem=1 if fp8 else 2)
     gates = None
     if args.workload == 5 and args.mode == "per_depth" and not fp8 and flags == 0 and not args.qk_norm \

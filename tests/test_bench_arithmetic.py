@@ -57,6 +57,8 @@ def test_traffic_records_are_well_formed(tmp_path, monkeypatch):
         assert e["dram_bytes_per_call"] > 0, key
         assert os.path.exists(os.path.join(bench.ROOT, e["profile"])), key
         assert len(e["kernel_hash"]) == 16, key
+        if key.startswith("w"):  # an attention record names the kernel it was captured on
+            assert e.get("kernel") in ("tcgen05", "m16n8k16"), key
         for name in e.get("sources", ()):
             assert os.path.exists(os.path.join(csrc, name)), (key, name)
     # a record is used only while its sources hash to its kernel_hash
@@ -64,11 +66,13 @@ def test_traffic_records_are_well_formed(tmp_path, monkeypatch):
     os.makedirs(fake_root / "profiles")
     os.symlink(os.path.join(bench.ROOT, "paper_2604_26412_gb300"), fake_root / "paper_2604_26412_gb300")
     good = {"kernel_hash": bench.kernel_source_hash(bench.MMA_SOURCES), "sources": list(bench.MMA_SOURCES),
-            "dram_bytes_per_call": 123.0, "how": "", "profile": ""}
+            "kernel": "m16n8k16", "dram_bytes_per_call": 123.0, "how": "", "profile": ""}
     stale = dict(good, kernel_hash="0" * 16)
     (fake_root / "profiles" / "traffic.json").write_text(json.dumps({"w5-per_depth": good, "w4-per_depth": stale}))
     monkeypatch.setattr(bench, "ROOT", str(fake_root))
     assert bench.recorded_traffic(5, "per_depth") == 123.0
+    assert bench.recorded_traffic(5, "per_depth", kernel="m16n8k16") == 123.0
+    assert bench.recorded_traffic(5, "per_depth", kernel="tcgen05") is None  # another kernel ran
     assert bench.recorded_traffic(4, "per_depth") is None
     assert bench.recorded_traffic(3, "per_depth") is None
 
