@@ -50,7 +50,6 @@ constexpr int kNK = 5;                     // K tiles in flight (freed when QK^T
 constexpr int kNV = 6;                     // V tiles in flight (freed when P.V completes)
 constexpr int kKVBytes = kKVTileBytes;     // one K or V tile
 constexpr int kNS = 4;                     // S buffers in TMEM: QK^T may run up to 4 tiles ahead of P.V
-constexpr int kNW = 2;                     // O accumulators: warpgroup w's tiles accumulate into O_w
 constexpr int kThreads = 12 * 32;
 constexpr int kProducerWarp = 10;          // K and V loads of even tiles
 constexpr int kProducerVWarp = 9;          // K and V loads of odd tiles, q blocks
@@ -185,7 +184,6 @@ struct Smem {
   uint64_t* sfull;     // [kNS]  S buffer written (QK^T completion)
   uint64_t* sfree;     // [kNS]  P.V of the tile in the S buffer completed: the buffer is free
   uint64_t* pfull;     // [kNS]  P written over the S buffer (the owning warpgroup's 128 threads)
-  uint64_t* pvdone;    // [kNW]  P.V into O_w of warpgroup w's latest tile completed
   uint64_t* ofree;     // [1]  epilogue finished reading O
   uint64_t* mmadone;   // [2]  every QK^T / every P.V completed
   uint64_t* full8;     // fp8 cache: [2][kLandSlots] codes landed (TMA)
@@ -206,7 +204,7 @@ struct Smem {
 __host__ __device__ inline size_t smem_bytes(int C, bool f8) {
   const int nk = f8 ? kF8NK : kNK, nv = f8 ? kF8NV : kNV;
   size_t off = static_cast<size_t>(nk + nv) * kKVBytes + kQBufBytes + (f8 ? 2 * kLandSlots * kLandBytes : 0);
-  off += sizeof(uint64_t) * (2 * nk + 2 * nv + 2 + 3 * kNS + kNW + 3 + 2 * kLandSlots + 3);
+  off += sizeof(uint64_t) * (2 * nk + 2 * nv + 2 + 3 * kNS + 3 + 2 * kLandSlots + 3);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(float) * 2 * kQRows;
   off += sizeof(uint32_t) * 4 + sizeof(int) * kMiscInts;
@@ -236,8 +234,7 @@ __device__ Smem carve(uint8_t* raw, int C, bool f8) {
   s.sfull = s.qempty + 1;
   s.sfree = s.sfull + kNS;
   s.pfull = s.sfree + kNS;
-  s.pvdone = s.pfull + kNS;
-  s.ofree = s.pvdone + kNW;
+  s.ofree = s.pfull + kNS;
   s.mmadone = s.ofree + 1;
   s.full8 = s.mmadone + 2;
   s.qland = s.full8 + 2 * kLandSlots;
@@ -305,7 +302,8 @@ __device__ __forceinline__ void run_mma_qk(const AttnParams& p, const Smem& sm, 
 // read from tensor memory (the tile's S columns).  Tile t needs its P and its
 // V tile; the first P.V into O_w of a piece (which overwrites O_w) needs the
 // previous piece's epilogue to have read O.  Each completion frees the tile's
-// S buffer for QK^T of tile t + kNS.
+// S buffer for QK^T of tile t + kNS and tells the softmax that O_w holds P.V
+// of tile t.
 template <bool kF8>
 __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                            Cursor cu) {
@@ -341,7 +339,6 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
       tc_mma_tmem_a(o, pcol + 8 * k16, bd, idesc, (first && k16 == 0) ? 0u : 1u);
     }
     tc_commit(smem_addr(&sm.vempty[t % NV]));
-    tc_commit(smem_addr(&sm.pvdone[t & 1]));
     tc_commit(smem_addr(&sm.sfree[t % kNS]));
   }
   tc_commit(smem_addr(&sm.mmadone[1]));
@@ -359,12 +356,15 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
 // 0..15, so every SM sub-partition's softmax warps get rows; two threads share
 // a lane (row), each with 32 of the 64 columns, and agree on the row max by
 // one shuffle.
-// O_wg *= alpha (per row) in TMEM, after P.V of this warpgroup's previous tile (t - 2) completed.
+// O_wg *= alpha (per row) in TMEM, after P.V of this warpgroup's previous tile (t - 2) completed:
+// sfree of its S buffer, which P.V commits when it completes.  A rescale needs an earlier tile of the
+// piece, so t >= 2, and the wait is unambiguous: S of tile t implies that P.V of tile t - 4 (and
+// so of t - 6) completed, and P.V of tile t + 2 cannot complete before this warpgroup's pfull of it.
 template <bool kSpread>
 __device__ __forceinline__ void rescale_o_tmem(const Smem& sm, const Pipe& pipe, const AttnParams& p, uint32_t my_o,
                                                int t, float alpha) {
   constexpr int kOChunks = kSpread ? 2 : 4;  // 32-column O chunks per thread
-  if (!mbar_wait(smem_addr(&sm.pvdone[t & 1]), ((t - 2) / kNW) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
+  if (!mbar_wait(smem_addr(&sm.sfree[(t - 2) % kNS]), ((t - 2) / kNS) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
   tc_fence_after();
 #pragma unroll
   for (int c = 0; c < kOChunks; ++c) {
@@ -538,12 +538,13 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         if constexpr (kSpread) tmem_st16x2_16(trow + sbuf * kTileKeys, pk);
         else tmem_st32(trow + sbuf * kTileKeys, pk);
       }
-      // P.V of this warpgroup's previous tile must complete before P of this tile is released: O_wg may
-      // then be rescaled, and pvdone never runs two phases ahead of this warpgroup's waits (S of this tile
-      // implies P.V of tile t - kNS; P.V of tile t needs the pfull below).
-      if (live && t >= kNW && !mbar_wait(smem_addr(&sm.pvdone[t & 1]), ((t - kNW) / kNW) & 1, p.err, p.wait_ns))
-        *pipe.abort = 1;
+      // Spread rows release P of this tile without waiting for P.V of this warpgroup's previous tile;
+      // only a rescale of O_wg waits for it (rescale_o_tmem).  Dense rows wait for it on every tile:
+      // releasing P earlier measured slower for them (whole-tree multi-layer tree 377 -> 384 us per
+      // call on GB300), while the spread rows gained 0.3-1%.
       if constexpr (!kSpread) {
+        if (live && t >= 2 && !mbar_wait(smem_addr(&sm.sfree[(t - 2) % kNS]), ((t - 2) / kNS) & 1, p.err, p.wait_ns))
+          *pipe.abort = 1;
         if (live && warp_live && any_rescale) rescale_o_tmem<kSpread>(sm, pipe, p, my_o, t, alpha);
       }
       if (live && warp_live) tmem_wait_st();
@@ -563,13 +564,14 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
     }
     if (ti.last) {
       // Every P.V of the piece has completed once P.V of tile t has (P.V
-      // completes in tile order).  The warpgroup that does not own tile t last
-      // waited P.V of tile t - 4, too far back to tell tile t's phase of pvdone
-      // from tile t - 6's by parity, so it first waits P.V of its own tile t - 1.
+      // completes in tile order; sfree of the tile's S buffer).  The owner of
+      // tile t saw S of it, so P.V of tile t - 4 had completed and the wait is
+      // unambiguous; the other warpgroup saw S of tile t - 1 only, so it first
+      // waits P.V of its own tile t - 1 (after which P.V of t - 4 has completed).
       bool ok = live;
       if (ok && (t & 1) != wg && t >= 1)
-        ok = mbar_wait(smem_addr(&sm.pvdone[(t - 1) & 1]), ((t - 1) / kNW) & 1, p.err, p.wait_ns);
-      ok = ok && mbar_wait(smem_addr(&sm.pvdone[t & 1]), (t / kNW) & 1, p.err, p.wait_ns);
+        ok = mbar_wait(smem_addr(&sm.sfree[(t - 1) % kNS]), ((t - 1) / kNS) & 1, p.err, p.wait_ns);
+      ok = ok && mbar_wait(smem_addr(&sm.sfree[t % kNS]), (t / kNS) & 1, p.err, p.wait_ns);
       ok = __all_sync(0xffffffffu, ok);
       tc_fence_after();
       float l_row = l_run;
@@ -1147,7 +1149,6 @@ struct SmemPair {
   uint64_t* sfull;     // [4]  S_{w,j} written (index 2 w + j)
   uint64_t* sfree;     // [4]  P.V of the tile in S_{w,j} completed: the buffer is free
   uint64_t* pfull;     // [4]  P_w of a tile with parity j written over S_{w,j} (128 threads)
-  uint64_t* pvdone;    // [2]  O_w += P_w V completed
   uint64_t* ofree;     // [2]  warpgroup w's epilogue read O_w (128 threads)
   uint64_t* mmadone;   // [4]  every MMA of an issuing thread completed (QK^T 0, 1, P.V 0, 1)
   uint64_t* anc;       // [64]
@@ -1160,7 +1161,7 @@ struct SmemPair {
 
 __host__ __device__ inline size_t smem_bytes_pair(int C) {
   size_t off = static_cast<size_t>(kPairNK + kPairNV) * kKVBytes + 2 * kQBufBytes;
-  off += sizeof(uint64_t) * (2 * kPairNK + 2 * kPairNV + 2 + 4 + 4 + 4 + 2 + 2 + 4);
+  off += sizeof(uint64_t) * (2 * kPairNK + 2 * kPairNV + 2 + 4 + 4 + 4 + 2 + 4);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(uint32_t) * 4 + sizeof(int) * kMiscInts;
   off += sizeof(int) * (2 * C + 1);
@@ -1186,8 +1187,7 @@ __device__ SmemPair carve_pair(uint8_t* raw, int C) {
   s.sfull = s.qempty + 1;
   s.sfree = s.sfull + 4;
   s.pfull = s.sfree + 4;
-  s.pvdone = s.pfull + 4;
-  s.ofree = s.pvdone + 2;
+  s.ofree = s.pfull + 4;
   s.mmadone = s.ofree + 2;
   s.anc = s.mmadone + 4;
   s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
@@ -1246,7 +1246,7 @@ __device__ __forceinline__ void run_mma_qk_pair(const AttnParams& p, const SmemP
 // with P_w read from tensor memory (the S columns of the tile).  The first P.V
 // into O_w of a piece (which overwrites O_w) needs the previous piece's
 // epilogue to have read O_w.  Each completion frees S buffer (w, t & 1) for
-// QK^T of tile t + 2.
+// QK^T of tile t + 2 and tells the softmax that O_w holds P.V of tile t.
 __device__ __forceinline__ void run_mma_pv_pair(const AttnParams& p, const SmemPair& sm, const Pipe& pipe,
                                                 uint32_t tmem, Cursor cu, int w) {
   constexpr uint32_t idesc = idesc_bf16(128, 128, true);
@@ -1278,7 +1278,6 @@ __device__ __forceinline__ void run_mma_pv_pair(const AttnParams& p, const SmemP
       const uint64_t bd = smem_desc_sw128(vbase + k16 * 2 * group_off, half_off, group_off);
       tc_mma_tmem_a(o, pcol + 8 * k16, bd, idesc, (t == piece_t0 && k16 == 0) ? 0u : 1u);
     }
-    tc_commit(smem_addr(&sm.pvdone[w]));
     tc_commit(smem_addr(&sm.sfree[2 * w + j]));
     tc_commit(smem_addr(&sm.vempty[t % kPairNV]));  // completes with both blocks' commits
   }
@@ -1383,12 +1382,16 @@ __device__ __forceinline__ void run_softmax_pair(const AttnParams& p, const Smem
       l_run += row_exp<kTileKeys, false>(pr, qscale, m_use, 1.f, pk);
       tmem_st32(my_s + j * kTileKeys, pk);  // P over the S columns just read
     }
-    // P.V of the previous tile must complete before P of this tile is released: O_wg may then be
-    // rescaled, and pvdone never runs two phases ahead of this warpgroup's waits (P.V of tile t needs
-    // the pfull below; S of this tile implies P.V of tile t - 2), so its parity stays unambiguous.
-    if (live && t > 0 && !mbar_wait(smem_addr(&sm.pvdone[wg]), (t - 1) & 1, p.err, p.wait_ns)) *pipe.abort = 1;
+    // Only a rescale of O_wg waits for P.V of the previous tile (sfree of its S buffer, which P.V
+    // commits when it completes); P of this tile is released without it, so that hand-off stays off
+    // the loop through the S buffers (whole-tree hybrid tree 83.3 -> 77.4 us per call on GB300).  A
+    // rescale needs an earlier tile of the piece, so t >= 1, and the wait is unambiguous: P.V of
+    // tile t - 3 completed before QK^T of tile t - 1 was issued, and P.V of tile t + 1 cannot
+    // complete before the pfull of tile t + 1.
     if (live && warp_live) {
       if (any_rescale) {  // O_wg *= alpha (P.V of this tile is issued only after pfull below)
+        if (!mbar_wait(smem_addr(&sm.sfree[2 * wg + ((t - 1) & 1)]), ((t - 1) >> 1) & 1, p.err, p.wait_ns))
+          *pipe.abort = 1;
         tc_fence_after();
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
@@ -1418,8 +1421,9 @@ __device__ __forceinline__ void run_softmax_pair(const AttnParams& p, const Smem
     tc_fence_before();
     mbar_arrive(smem_addr(&sm.pfull[2 * wg + j]));
     if (ti.last) {
-      // Every P.V of the piece has completed once P.V of tile t has (P.V of tile t - 1 was waited above).
-      bool ok = live && mbar_wait(smem_addr(&sm.pvdone[wg]), t & 1, p.err, p.wait_ns);
+      // Every P.V of the piece has completed once P.V of tile t has (they complete in order; the
+      // parity is unambiguous as for the rescale wait above).
+      bool ok = live && mbar_wait(smem_addr(&sm.sfree[2 * wg + (t & 1)]), (t >> 1) & 1, p.err, p.wait_ns);
       ok = __all_sync(0xffffffffu, ok);
       tc_fence_after();
       if (ok && warp_live) {
@@ -1495,10 +1499,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       mbar_init(smem_addr(&sm.pfull[b]), kQRows);
       mbar_init(smem_addr(&sm.mmadone[b]), 1);
     }
-    for (int w = 0; w < 2; ++w) {
-      mbar_init(smem_addr(&sm.pvdone[w]), 1);
-      mbar_init(smem_addr(&sm.ofree[w]), kQRows);
-    }
+    for (int w = 0; w < 2; ++w) mbar_init(smem_addr(&sm.ofree[w]), kQRows);
     for (int i = 0; i < kMiscInts; ++i) sm.misc[i] = 0;
     fence_mbar_init();
     prefetch_tensormap(&maps.tk);
@@ -1589,7 +1590,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_addr(&sm.sfree[b]), 1);
       mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads / 2);
     }
-    for (int w = 0; w < kNW; ++w) mbar_init(smem_addr(&sm.pvdone[w]), 1);
     if constexpr (kF8) {
       for (int l = 0; l < 2 * kLandSlots; ++l) mbar_init(smem_addr(&sm.full8[l]), 1);
       mbar_init(smem_addr(sm.qland), 1);
