@@ -557,8 +557,8 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
           const int key = ti.nkeys + (i >> 4), ch = i & 15;
           *reinterpret_cast<uint4*>(vptr + tile_off_tc(key, ch, ti.draft || p.prefix_grouped)) = make_uint4(0, 0, 0, 0);
         }
+        fence_proxy_async_smem();  // the zeros, written through the generic proxy, are read by P.V
       }
-      fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(smem_addr(&sm.pfull[sbuf]));
     }
