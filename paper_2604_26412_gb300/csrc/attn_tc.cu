@@ -65,7 +65,9 @@ constexpr int kMiscInts = 20;
 constexpr int kF8NK = 3;
 constexpr int kF8NV = 4;
 constexpr int kLandBytes = 2 * kTileKeys * 128;  // one landing slot: a tile's K codes then its V codes
-constexpr int kLandSlots = 2;                    // per producer warp: one own tile in flight, one decoding
+constexpr int kLandSlots = 4;                    // tile t lands in slot t % 4, freed when it is decoded
+constexpr int kDecodeAhead = 3;                  // the softmax warpgroup done with tile t decodes tile t + 3
+constexpr int kBarDecode0 = 2;                   // named barriers 2, 3: the 128 threads of warpgroup 0, 1
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max grows by > 256x
 
 // Row modes.  Dense: one block of up to 128 stacked rows, one thread per TMEM lane, the two
@@ -174,7 +176,7 @@ struct Smem {
   uint8_t* kring;      // kNK x K tile
   uint8_t* vring;      // kNV x V tile
   uint8_t* qbuf;       // one q block
-  uint8_t* land;       // fp8 cache: [2 producer warps][kLandSlots] landing slots of e4m3 codes
+  uint8_t* land;       // fp8 cache: [kLandSlots] landing slots of e4m3 codes (K codes, then V codes)
   uint64_t* kfull;     // [kNK]  TMA -> MMA
   uint64_t* kempty;    // [kNK]  QK^T of the slot's tile completed -> TMA
   uint64_t* vfull;     // [kNV]  TMA -> MMA, softmax
@@ -186,7 +188,8 @@ struct Smem {
   uint64_t* pfull;     // [kNS]  P written over the S buffer (the owning warpgroup's 128 threads)
   uint64_t* ofree;     // [1]  epilogue finished reading O
   uint64_t* mmadone;   // [2]  every QK^T / every P.V completed
-  uint64_t* full8;     // fp8 cache: [2][kLandSlots] codes landed (TMA)
+  uint64_t* lfull;     // fp8 cache: [kLandSlots] the tile's codes landed (TMA), or a draft tile passed through
+  uint64_t* lfree;     // fp8 cache: [kLandSlots] the tile in the slot was decoded: the slot is free
   uint64_t* qland;     // fp8 cache: [1] bf16 q block landed (converted to f16 before qfull)
   uint64_t* dland;     // fp8 cache: [2] a producer warp's bf16 draft tile landed (converted before kfull / vfull)
   uint64_t* anc;       // [64]
@@ -194,21 +197,23 @@ struct Smem {
   float* comb;         // [128][2] second warpgroup's (max, sum) per row at a piece end
   uint32_t* tmem_base;
   int* misc;           // [0] abort, [2] K tiles consumed, [3]/[4] q blocks issued/consumed, [6] V tiles consumed,
-                       // [8..9] / [10..11] K / V tiles issued per producer warp, [12..13] / [14..15] fp8 landings
-                       // issued / decoded per producer warp, [1] fp8: q blocks converted, [16..17] / [18..19] fp8:
-                       // draft tiles landed / converted per producer warp
+                       // [8..9] / [10..11] K / V tiles issued per producer warp, [12..13] fp8: tiles of
+                       // parity 0 / 1 whose landing was issued, [14..15] fp8: of those, tiles whose landing a
+                       // decoder waited, [1] fp8: q blocks converted, [16..17] / [18..19] fp8: draft tiles
+                       // landed / converted per producer warp
   int* len;
   int* base;
+  int* lkind;          // fp8 cache: [kLandSlots] 1 when the slot's tile is a draft tile (nothing to decode)
 };
 
 __host__ __device__ inline size_t smem_bytes(int C, bool f8) {
   const int nk = f8 ? kF8NK : kNK, nv = f8 ? kF8NV : kNV;
-  size_t off = static_cast<size_t>(nk + nv) * kKVBytes + kQBufBytes + (f8 ? 2 * kLandSlots * kLandBytes : 0);
+  size_t off = static_cast<size_t>(nk + nv) * kKVBytes + kQBufBytes + (f8 ? kLandSlots * kLandBytes : 0);
   off += sizeof(uint64_t) * (2 * nk + 2 * nv + 2 + 3 * kNS + 3 + 2 * kLandSlots + 3);
   off += sizeof(uint64_t) * kMaxTreeNodes + sizeof(int) * kMaxTreeNodes;
   off += sizeof(float) * 2 * kQRows;
   off += sizeof(uint32_t) * 4 + sizeof(int) * kMiscInts;
-  off += sizeof(int) * (2 * C + 1);
+  off += sizeof(int) * (2 * C + 1) + sizeof(int) * kLandSlots;
   return off + 1024;
 }
 
@@ -223,7 +228,7 @@ __device__ Smem carve(uint8_t* raw, int C, bool f8) {
   s.qbuf = p;
   p += kQBufBytes;
   s.land = p;
-  if (f8) p += 2 * kLandSlots * kLandBytes;
+  if (f8) p += kLandSlots * kLandBytes;
   uint64_t* b = reinterpret_cast<uint64_t*>(p);
   s.kfull = b;
   s.kempty = s.kfull + nk;
@@ -236,8 +241,9 @@ __device__ Smem carve(uint8_t* raw, int C, bool f8) {
   s.pfull = s.sfree + kNS;
   s.ofree = s.pfull + kNS;
   s.mmadone = s.ofree + 1;
-  s.full8 = s.mmadone + 2;
-  s.qland = s.full8 + 2 * kLandSlots;
+  s.lfull = s.mmadone + 2;
+  s.lfree = s.lfull + kLandSlots;
+  s.qland = s.lfree + kLandSlots;
   s.dland = s.qland + 1;
   s.anc = s.dland + 2;
   s.par = reinterpret_cast<int*>(s.anc + kMaxTreeNodes);
@@ -246,6 +252,7 @@ __device__ Smem carve(uint8_t* raw, int C, bool f8) {
   s.misc = reinterpret_cast<int*>(s.tmem_base + 4);
   s.len = s.misc + kMiscInts;
   s.base = s.len + C;
+  s.lkind = s.base + C + 1;
   return s;
 }
 
@@ -344,6 +351,43 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
   tc_commit(smem_addr(&sm.mmadone[1]));
 }
 
+// e4m3 codes of one landed K or V tile ([64 rows][128 codes], 128-byte swizzle) -> f16 in the grouped
+// layout, one hardware conversion per two codes (exact: 3 mantissa bits, exponents within f16's
+// normal range); the power-of-two scales are applied by the consumers.  The four warps of a
+// warpgroup share a tile: warp w decodes key rows 16 w .. 16 w + 15 (8-row groups 2 w, 2 w + 1).
+// Lane l takes 16-byte chunk c = l & 7 (dims 16c..16c+15) of rows 16 w + 4 i + (l >> 3), i = 0..3:
+// rows 8k + r0 (even i) and 8k + 4 + r0 (odd i) take fixed swizzles, so every address is one of
+// four per-lane bases plus a constant.  The four loads go out before any conversion or store, so
+// that their latencies overlap.
+__device__ __forceinline__ void decode_e4m3_quarter(uint32_t src, uint32_t dst, int lane, int w) {
+  const uint32_t c = lane & 7, r0 = lane >> 3;
+  const uint32_t s_even = src + r0 * 128 + ((c ^ r0) << 4);
+  const uint32_t s_odd = src + (r0 + 4) * 128 + ((c ^ (r0 + 4)) << 4);
+  const uint32_t dh = (c >> 2) * kGroupHalfBytes;
+  const uint32_t d_even0 = dst + dh + r0 * 128 + ((((2 * c) & 7) ^ r0) << 4);
+  const uint32_t d_even1 = dst + dh + r0 * 128 + ((((2 * c + 1) & 7) ^ r0) << 4);
+  const uint32_t d_odd0 = dst + dh + (r0 + 4) * 128 + ((((2 * c) & 7) ^ (r0 + 4)) << 4);
+  const uint32_t d_odd1 = dst + dh + (r0 + 4) * 128 + ((((2 * c + 1) & 7) ^ (r0 + 4)) << 4);
+  const uint32_t k0 = 2 * static_cast<uint32_t>(w);
+  uint4 v[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) v[i] = lds128((i & 1 ? s_odd : s_even) + (k0 + (i >> 1)) * 1024);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t k = k0 + (i >> 1);
+    const uint32_t ws[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+    uint32_t o[8];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %2;\n\t"
+          "cvt.rn.f16x2.e4m3x2 %0, lo;\n\tcvt.rn.f16x2.e4m3x2 %1, hi;\n\t}"
+          : "=r"(o[2 * q]), "=r"(o[2 * q + 1])
+          : "r"(ws[q]));
+    sts128((i & 1 ? d_odd0 : d_even0) + k * kGroupBytes, make_uint4(o[0], o[1], o[2], o[3]));
+    sts128((i & 1 ? d_odd1 : d_even1) + k * kGroupBytes, make_uint4(o[4], o[5], o[6], o[7]));
+  }
+}
+
 // ------------------------------------------------------------ softmax + epilogue
 
 // Tile ownership: warpgroup w takes the tiles t with t % 2 == w (all 64 keys)
@@ -383,7 +427,7 @@ __device__ __forceinline__ void rescale_o_tmem(const Smem& sm, const Pipe& pipe,
 template <bool kSpread, bool kF8>
 __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm, const Pipe& pipe, uint32_t tmem,
                                             Cursor cu) {
-  constexpr int NV = kF8 ? kF8NV : kNV;
+  constexpr int NK = kF8 ? kF8NK : kNK, NV = kF8 ? kF8NV : kNV;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int quarter = warp & 3;                 // TMEM lanes this warp may access
   const int wg = warp >> 2;                     // warpgroup: owns tiles t with t % 2 == wg
@@ -408,9 +452,48 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
   bool valid = false, warp_live = false;
   float m_run = -INFINITY, l_run = 0.f;  // l_run: this thread's columns only (spread)
   int t = 0, anc_seq = -1;
+  // fp8 cache: decodes tile y (its codes landed in slot y % kLandSlots) into its K and V ring slots with
+  // this warpgroup's 128 threads, or passes a draft tile's landing through (its producer warp filled
+  // the rings).  Tile y is decoded by warpgroup (y + 1) % 2 once it is done with tile y - kDecodeAhead
+  // (its own tile; tiles 0..2 before the loop), so QK^T of tile y never waits for the warpgroup that
+  // will take its softmax.  The ring-slot waits are unambiguous: that warpgroup has seen S of tile
+  // y - 3, so QK^T of tile y - 2 NK and P.V of tile y - 2 NV had completed.
+  const int ntiles = cu.t_end - cu.t_begin;
+  auto decode_landed = [&](int y) {
+    const int ls = y % kLandSlots;
+    bool good = !*pipe.abort && mbar_wait(smem_addr(&sm.lfull[ls]), (y / kLandSlots) & 1, p.err, p.wait_ns);
+    const bool landed = good;
+    const bool codes = good && sm.lkind[ls] == 0;
+    if (codes) {
+      good = mbar_wait(smem_addr(&sm.kempty[y % NK]), ((y / NK) & 1) ^ 1u, p.err, p.wait_ns) &&
+             mbar_wait(smem_addr(&sm.vempty[y % NV]), ((y / NV) & 1) ^ 1u, p.err, p.wait_ns);
+      if (good) {
+        const uint32_t src = smem_addr(sm.land + static_cast<size_t>(ls) * kLandBytes);
+        decode_e4m3_quarter(src, smem_addr(sm.kring + static_cast<size_t>(y % NK) * kKVBytes), lane, quarter);
+        decode_e4m3_quarter(src + kLandBytes / 2, smem_addr(sm.vring + static_cast<size_t>(y % NV) * kKVBytes),
+                            lane, quarter);
+        fence_proxy_async_smem();  // the MMAs read the tiles through the async proxy
+      }
+    }
+    if (!good) *pipe.abort = 1;
+    named_barrier_sync(kBarDecode0 + wg, kSoftmaxThreads / 2);
+    if (wtid == 0) {
+      if (codes && good) {
+        mbar_arrive(smem_addr(&sm.kfull[y % NK]));
+        mbar_arrive(smem_addr(&sm.vfull[y % NV]));
+      }
+      if (landed) {
+        mbar_arrive(smem_addr(&sm.lfree[ls]));
+        sm.misc[14 + (y & 1)] = (y >> 1) + 1;
+      }
+    }
+  };
   // Outputs and the workspace are written only once the preceding kernel has ended
   // (KVSHOT_OVERLAP_PREVIOUS); the first S needs q, which comes after that anyway.
   wait_for_prerequisite_grid();
+  if constexpr (kF8) {
+    for (int y = 1 - wg; y < min(kDecodeAhead, ntiles); y += 2) decode_landed(y);
+  }
   for (; cu.t < cu.t_end; cursor_next(cu, p, sm.len)) {
     const TileInfo ti = tile_info(cu, p);
     if (cu.c != unit_c || cu.hr != unit_hr) {
@@ -561,6 +644,9 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
       }
       tc_fence_before();
       mbar_arrive(smem_addr(&sm.pfull[sbuf]));
+      if constexpr (kF8) {
+        if (t + kDecodeAhead < ntiles) decode_landed(t + kDecodeAhead);
+      }
     }
     if (ti.last) {
       // Every P.V of the piece has completed once P.V of tile t has (P.V
@@ -891,132 +977,26 @@ __device__ __forceinline__ TileBoxes tile_boxes_f8(const AttnParams& p, const Cu
   return tb;
 }
 
-// e4m3 codes of one landed K or V tile ([64 rows][128 codes], 128-byte swizzle) -> f16 in the grouped
-// layout, one hardware conversion per two codes (exact: 3 mantissa bits, exponents within f16's
-// normal range); the power-of-two scales are applied by the consumers.  Lane = one 16-code chunk of a
-// row per step (a warp reads 4 whole rows per step).
-__device__ __forceinline__ void decode_e4m3_tile(uint32_t src, uint32_t dst, int lane) {
-  // Lane l decodes 16-byte chunk c = l & 7 (dims 16c..16c+15) of key rows r = 4 it + (l >> 3), it = 0..15.
-  // Rows 8k + r0 (even it) and 8k + 4 + r0 (odd it) take fixed swizzles, so every address is one of four
-  // per-lane bases plus a constant.  The loads go out in batches of sixteen before any conversion or
-  // store, so that their latencies overlap (one load per iteration measured ~100 cycles per iteration).
-  const uint32_t c = lane & 7, r0 = lane >> 3;
-  const uint32_t s_even = src + r0 * 128 + ((c ^ r0) << 4);
-  const uint32_t s_odd = src + (r0 + 4) * 128 + ((c ^ (r0 + 4)) << 4);
-  const uint32_t dh = (c >> 2) * kGroupHalfBytes;
-  const uint32_t d_even0 = dst + dh + r0 * 128 + ((((2 * c) & 7) ^ r0) << 4);
-  const uint32_t d_even1 = dst + dh + r0 * 128 + ((((2 * c + 1) & 7) ^ r0) << 4);
-  const uint32_t d_odd0 = dst + dh + (r0 + 4) * 128 + ((((2 * c) & 7) ^ (r0 + 4)) << 4);
-  const uint32_t d_odd1 = dst + dh + (r0 + 4) * 128 + ((((2 * c + 1) & 7) ^ (r0 + 4)) << 4);
-  constexpr int kIters = kTileKeys * 8 / 32, kBatch = 16;
-#pragma unroll
-  for (int b0 = 0; b0 < kIters; b0 += kBatch) {
-    uint4 w[kBatch];
-#pragma unroll
-    for (int i = 0; i < kBatch; ++i) {
-      const int it = b0 + i;
-      w[i] = lds128((it & 1 ? s_odd : s_even) + static_cast<uint32_t>(it >> 1) * 1024);
-    }
-#pragma unroll
-    for (int i = 0; i < kBatch; ++i) {
-      const int it = b0 + i;
-      const uint32_t k = static_cast<uint32_t>(it >> 1);
-      const uint32_t ws[4] = {w[i].x, w[i].y, w[i].z, w[i].w};
-      uint32_t o[8];
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %2;\n\t"
-            "cvt.rn.f16x2.e4m3x2 %0, lo;\n\tcvt.rn.f16x2.e4m3x2 %1, hi;\n\t}"
-            : "=r"(o[2 * q]), "=r"(o[2 * q + 1])
-            : "r"(ws[q]));
-      sts128((it & 1 ? d_odd0 : d_even0) + k * kGroupBytes, make_uint4(o[0], o[1], o[2], o[3]));
-      sts128((it & 1 ? d_odd1 : d_even1) + k * kGroupBytes, make_uint4(o[4], o[5], o[6], o[7]));
-    }
-  }
-}
-
-// Producer warp `role` with an fp8 target cache.  For each of its tiles (t % 2 == role) it first lands
-// the codes of a prefix tile in its own slot (the n-th landing -> slot n % 2, one own tile ahead), then
-// finishes its oldest pending own tile: once that tile's K and V ring slots are free it decodes the landed
-// codes into them and arrives on kfull / vfull, or, for a draft tile (bf16), issues its loads straight
-// into the rings.  q blocks as in run_producer_tc (role 1).
+// Producer warp `role` with an fp8 target cache; its tiles are t % 2 == role.  A prefix tile's e4m3
+// codes land in landing slot t % kLandSlots once the decode of tile t - kLandSlots has freed it; the
+// softmax warpgroups decode them into the f16 ring tiles (decode_landed in run_softmax), which keeps
+// the decode (and its shared-memory traffic) off this warp, whose box issues and waits then bound
+// nothing.  A draft tile (bf16) is loaded straight into its ring slots and converted to f16 in place
+// here, and its landing slot is passed through (lkind 1) so that every tile takes one phase of its
+// slot's barriers.  q blocks as in run_producer_tc (role 1), converted to f16 here.
 __device__ __forceinline__ void run_producer_f8(const AttnParams& p, const TensorMaps& maps, const Smem& sm,
                                                 const Pipe& pipe, Cursor cu, int nq_box, int role) {
   constexpr int NK = kF8NK, NV = kF8NV;
   const int lane = threadIdx.x & 31;
   const uint64_t policy = l2_policy_evict_first();
   PageWindow win;
-  int t = 0, piece = 0, landed = 0;  // landed: prefix tiles whose codes this warp has landed
+  int t = 0, piece = 0;
   const bool small = p.len_bound < (1 << 24) - 2 * kTileKeys;
   const FastDiv pdiv(p.paged ? p.page_size : 1, small), rbdiv(p.row_blocks, true);
   int unit_c = -1, unit_hr = -1, h = 0, pages = 0;
   int ok = 1;
   bool waited = false;
-  int drafts = 0, qblocks = 0;  // draft tiles this warp landed, q blocks it loaded
-  // Own tiles whose rings are not filled yet (oldest first, at most kLandSlots - 1): tile index,
-  // landing index (prefix tiles) and boxes.
-  constexpr int kPend = kLandSlots - 1;
-  int npend = 0, pend_t[kPend], pend_land[kPend];
-  TileBoxes pend_tb[kPend];
-  uint8_t* land = sm.land + static_cast<size_t>(role) * kLandSlots * kLandBytes;
-  // Fills the K and V ring slots of own tile x (boxes tb; a prefix tile's codes are landing jx).
-  auto finish = [&](int x, int jx, const TileBoxes& tb) -> bool {
-    const int kslot = x % NK, vslot = x % NV;
-    int good = 1;
-    if (lane < 2) {
-      const uint32_t bar = lane == 0 ? smem_addr(&sm.kempty[kslot]) : smem_addr(&sm.vempty[vslot]);
-      const uint32_t par = ((x / (lane == 0 ? NK : NV)) & 1) ^ 1u;
-      good = mbar_wait(bar, par, p.err, p.wait_ns) && !*pipe.abort;
-    }
-    if (!__all_sync(0xffffffffu, good)) return false;
-    uint8_t* kd = sm.kring + static_cast<size_t>(kslot) * kKVBytes;
-    uint8_t* vd = sm.vring + static_cast<size_t>(vslot) * kKVBytes;
-    if (tb.draft) {
-      if (!waited) {  // the draft K/V may come from the preceding kernel (KVSHOT_OVERLAP_PREVIOUS)
-        wait_for_prerequisite_grid();
-        waited = true;
-      }
-      // bf16 draft K/V land in the ring slots and are converted to f16 there.
-      const int kv = lane >> 4, i = lane & 15;
-      const uint32_t dbar = smem_addr(&sm.dland[role]);
-      if (lane == 0) mbar_arrive_expect_tx(dbar, 2 * tb.bytes);
-      __syncwarp();
-      if (i < tb.nbox) tma_load_3d(smem_addr(kv ? vd : kd) + tb.off, kv ? &maps.dv : &maps.dk, 0, tb.y, 0, dbar,
-                                   policy);
-      if (lane == 0) sm.misc[16 + role] = drafts + 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(dbar, drafts & 1, p.err, p.wait_ns))) return false;
-      ++drafts;
-      bf16_to_f16_inplace(smem_addr(kd), kKVBytes, lane);
-      bf16_to_f16_inplace(smem_addr(vd), kKVBytes, lane);
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(smem_addr(&sm.kfull[kslot]));
-        mbar_arrive(smem_addr(&sm.vfull[vslot]));
-        sm.misc[18 + role] = drafts;
-      }
-    } else {
-      const int sl = jx % kLandSlots;
-      if (!mbar_wait(smem_addr(&sm.full8[role * kLandSlots + sl]), (jx / kLandSlots) & 1, p.err, p.wait_ns))
-        good = 0;
-      if (!__all_sync(0xffffffffu, good)) return false;
-      const uint32_t src = smem_addr(land + static_cast<size_t>(sl) * kLandBytes);
-      decode_e4m3_tile(src, smem_addr(kd), lane);
-      decode_e4m3_tile(src + kLandBytes / 2, smem_addr(vd), lane);
-      fence_proxy_async_smem();  // the MMAs read the tiles through the async proxy; the slot is reloaded by TMA
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(smem_addr(&sm.kfull[kslot]));
-        mbar_arrive(smem_addr(&sm.vfull[vslot]));
-        sm.misc[14 + role] = jx + 1;
-      }
-    }
-    if (lane == 0) {
-      sm.misc[8 + role] = x + 1;
-      sm.misc[10 + role] = x + 1;
-    }
-    return true;
-  };
+  int drafts = 0, qblocks = 0, issued = 0;  // draft tiles loaded, q blocks converted, own tiles issued
   for (; cu.t < cu.t_end; ++t, cursor_next(cu, p, sm.len)) {
     const bool first = cu.t == cu.t_begin || cu.lt == 0;  // first tile of a piece
     const bool mine = (t & 1) == role;
@@ -1030,17 +1010,7 @@ __device__ __forceinline__ void run_producer_f8(const AttnParams& p, const Tenso
       h = rbdiv.div(cu.hr);
       pages = p.paged ? pdiv.div(cu.L + p.page_size - 1) : 0;
     }
-    if (first && role == 1) {  // the unit's q block
-      // The q buffer is released by QK^T of the previous piece's last tile, which may be this warp's
-      // pending tile: finish it before waiting.
-      bool good = true;
-      for (int k = 0; k < npend && good; ++k) good = finish(pend_t[k], pend_land[k], pend_tb[k]);
-      npend = 0;
-      if (!good) {
-        if (lane == 0) *pipe.abort = 1;
-        ok = 0;
-        break;
-      }
+    if (first && role == 1) {  // the unit's q block (released by QK^T of the previous piece's last tile)
       if (!waited) {
         wait_for_prerequisite_grid();
         waited = true;
@@ -1085,42 +1055,73 @@ __device__ __forceinline__ void run_producer_f8(const AttnParams& p, const Tenso
     const bool draft = cu.lt >= cu.pt;
     const TileBoxes tb = draft ? tile_boxes(p, cu, win, lane, h, pages, pdiv) : tile_boxes_f8(p, cu, win, lane, h,
                                                                                                 pages, pdiv);
-    if (!draft) {  // land the codes: landing n -> slot n % 2, free since landing n - 2 (an earlier tile) was decoded
-      const int sl = landed % kLandSlots;
-      const uint32_t fbar = smem_addr(&sm.full8[role * kLandSlots + sl]);
-      uint8_t* dst = land + static_cast<size_t>(sl) * kLandBytes;
-      const int kv = lane >> 4, i = lane & 15;
-      if ((lane & 15) == 0 && kv == 0) mbar_arrive_expect_tx(fbar, 2 * tb.bytes);
-      __syncwarp();
-      if (i < tb.nbox)
-        tma_load_2d(smem_addr(dst + kv * (kLandBytes / 2)) + tb.off, kv ? &maps.tv : &maps.tk, 0, tb.y, fbar, policy);
-      if (lane == 0) sm.misc[12 + role] = landed + 1;
+    const int ls = t % kLandSlots;
+    const uint32_t lbar = smem_addr(&sm.lfull[ls]);
+    // The landing slot is free once tile t - kLandSlots (this warp's, two own tiles back) was decoded.
+    if (lane == 0)
+      ok = mbar_wait(smem_addr(&sm.lfree[ls]), ((t / kLandSlots) & 1) ^ 1u, p.err, p.wait_ns) && !*pipe.abort;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (!ok) {
+      if (lane == 0) *pipe.abort = 1;
+      break;
     }
-    if (npend == kPend) {  // the oldest pending tile, whose codes have had the longest to land
-      if (!finish(pend_t[0], pend_land[0], pend_tb[0])) {
+    const int kv = lane >> 4, i = lane & 15;
+    if (draft) {
+      const int kslot = t % NK, vslot = t % NV;
+      int good = 1;
+      if (lane < 2) {
+        const uint32_t bar = lane == 0 ? smem_addr(&sm.kempty[kslot]) : smem_addr(&sm.vempty[vslot]);
+        const uint32_t par = ((t / (lane == 0 ? NK : NV)) & 1) ^ 1u;
+        good = mbar_wait(bar, par, p.err, p.wait_ns) && !*pipe.abort;
+      }
+      if (!__all_sync(0xffffffffu, good)) {
         ok = 0;
         if (lane == 0) *pipe.abort = 1;
         break;
       }
-#pragma unroll
-      for (int k = 1; k < kPend; ++k) {
-        pend_t[k - 1] = pend_t[k];
-        pend_land[k - 1] = pend_land[k];
-        pend_tb[k - 1] = pend_tb[k];
+      if (!waited) {  // the draft K/V may come from the preceding kernel (KVSHOT_OVERLAP_PREVIOUS)
+        wait_for_prerequisite_grid();
+        waited = true;
       }
-      --npend;
+      // bf16 draft K/V land in the ring slots and are converted to f16 there.
+      uint8_t* kd = sm.kring + static_cast<size_t>(kslot) * kKVBytes;
+      uint8_t* vd = sm.vring + static_cast<size_t>(vslot) * kKVBytes;
+      const uint32_t dbar = smem_addr(&sm.dland[role]);
+      if (lane == 0) mbar_arrive_expect_tx(dbar, 2 * tb.bytes);
+      __syncwarp();
+      if (i < tb.nbox) tma_load_3d(smem_addr(kv ? vd : kd) + tb.off, kv ? &maps.dv : &maps.dk, 0, tb.y, 0, dbar,
+                                   policy);
+      if (lane == 0) sm.misc[16 + role] = drafts + 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(dbar, drafts & 1, p.err, p.wait_ns))) {
+        ok = 0;
+        if (lane == 0) *pipe.abort = 1;
+        break;
+      }
+      ++drafts;
+      bf16_to_f16_inplace(smem_addr(kd), kKVBytes, lane);
+      bf16_to_f16_inplace(smem_addr(vd), kKVBytes, lane);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(smem_addr(&sm.kfull[kslot]));
+        mbar_arrive(smem_addr(&sm.vfull[vslot]));
+        sm.misc[18 + role] = drafts;
+        sm.lkind[ls] = 1;  // released by the arrive below
+        mbar_arrive(lbar);
+      }
+    } else {
+      // The codes: K boxes from lanes 0..15, V boxes from lanes 16..31, rows at 128 bytes in order.
+      if (lane == 0) {
+        sm.lkind[ls] = 0;  // released by the arrive below
+        mbar_arrive_expect_tx(lbar, 2 * tb.bytes);
+      }
+      __syncwarp();
+      uint8_t* dst = sm.land + static_cast<size_t>(ls) * kLandBytes + kv * (kLandBytes / 2);
+      if (i < tb.nbox) tma_load_2d(smem_addr(dst) + tb.off, kv ? &maps.tv : &maps.tk, 0, tb.y, lbar, policy);
     }
-    pend_t[npend] = t;
-    pend_land[npend] = landed;
-    pend_tb[npend] = tb;
-    ++npend;
-    landed += draft ? 0 : 1;
+    ++issued;
+    if (lane == 0) sm.misc[12 + role] = issued;
   }
-  for (int k = 0; ok && k < npend; ++k)
-    if (!finish(pend_t[k], pend_land[k], pend_tb[k])) {
-      ok = 0;
-      if (lane == 0) *pipe.abort = 1;
-    }
 }
 
 // ============================================================ paired row blocks
@@ -1591,7 +1592,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_addr(&sm.pfull[b]), kSoftmaxThreads / 2);
     }
     if constexpr (kF8) {
-      for (int l = 0; l < 2 * kLandSlots; ++l) mbar_init(smem_addr(&sm.full8[l]), 1);
+      for (int l = 0; l < kLandSlots; ++l) {
+        mbar_init(smem_addr(&sm.lfull[l]), 1);
+        mbar_init(smem_addr(&sm.lfree[l]), 1);
+      }
       mbar_init(smem_addr(sm.qland), 1);
       mbar_init(smem_addr(&sm.dland[0]), 1);
       mbar_init(smem_addr(&sm.dland[1]), 1);
@@ -1653,9 +1657,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int k = sm.misc[1]; k < sm.misc[3]; ++k)
         if (!mbar_wait(smem_addr(sm.qland), k & 1, p.err)) break;
       for (int role = 0; role < 2; ++role) {
-        for (int j = sm.misc[14 + role]; j < sm.misc[12 + role]; ++j)
-          if (!mbar_wait(smem_addr(&sm.full8[role * kLandSlots + j % kLandSlots]), (j / kLandSlots) & 1, p.err))
-            break;
+        for (int j = sm.misc[14 + role]; j < sm.misc[12 + role]; ++j) {  // tile role + 2 j
+          const int y = role + 2 * j;
+          if (!mbar_wait(smem_addr(&sm.lfull[y % kLandSlots]), (y / kLandSlots) & 1, p.err)) break;
+        }
         for (int j = sm.misc[18 + role]; j < sm.misc[16 + role]; ++j)
           if (!mbar_wait(smem_addr(&sm.dland[role]), j & 1, p.err)) break;
       }
