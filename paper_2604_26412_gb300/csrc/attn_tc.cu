@@ -68,6 +68,7 @@ constexpr int kLandBytes = 2 * kTileKeys * 128;  // one landing slot: a tile's K
 constexpr int kLandSlots = 4;                    // tile t lands in slot t % 4, freed when it is decoded
 constexpr int kDecodeAhead = 3;                  // the softmax warpgroup done with tile t decodes tile t + 3
 constexpr int kBarDecode0 = 2;                   // named barriers 2, 3: the 128 threads of warpgroup 0, 1
+static_assert(kLandSlots % 2 == 0, "a landing slot must stay with one producer warp (t and t - kLandSlots)");
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when the max grows by > 256x
 
 // Row modes.  Dense: one block of up to 128 stacked rows, one thread per TMEM lane, the two
@@ -1058,6 +1059,9 @@ __device__ __forceinline__ void run_producer_f8(const AttnParams& p, const Tenso
     const int ls = t % kLandSlots;
     const uint32_t lbar = smem_addr(&sm.lfull[ls]);
     // The landing slot is free once tile t - kLandSlots (this warp's, two own tiles back) was decoded.
+    // The wait is unambiguous because kLandSlots is even: the slot's previous release, the decode of
+    // tile t - 2 kLandSlots, was waited by this warp before it landed tile t - kLandSlots.  (With an
+    // odd count the slot alternates between the two warps and this wait could pass two phases early.)
     if (lane == 0)
       ok = mbar_wait(smem_addr(&sm.lfree[ls]), ((t / kLandSlots) & 1) ^ 1u, p.err, p.wait_ns) && !*pipe.abort;
     ok = __shfl_sync(0xffffffffu, ok, 0);
