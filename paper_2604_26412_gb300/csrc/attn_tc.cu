@@ -352,30 +352,33 @@ __device__ __forceinline__ void run_mma_pv(const AttnParams& p, const Smem& sm, 
   tc_commit(smem_addr(&sm.mmadone[1]));
 }
 
-// e4m3 codes of one landed K or V tile ([64 rows][128 codes], 128-byte swizzle) -> f16 in the grouped
-// layout, one hardware conversion per two codes (exact: 3 mantissa bits, exponents within f16's
-// normal range); the power-of-two scales are applied by the consumers.  The four warps of a
-// warpgroup share a tile: warp w decodes key rows 16 w .. 16 w + 15 (8-row groups 2 w, 2 w + 1).
-// Lane l takes 16-byte chunk c = l & 7 (dims 16c..16c+15) of rows 16 w + 4 i + (l >> 3), i = 0..3:
-// rows 8k + r0 (even i) and 8k + 4 + r0 (odd i) take fixed swizzles, so every address is one of
-// four per-lane bases plus a constant.  The four loads go out before any conversion or store, so
-// that their latencies overlap.
-__device__ __forceinline__ void decode_e4m3_quarter(uint32_t src, uint32_t dst, int lane, int w) {
+// e4m3 codes of one landed tile ([64 rows][128 codes] of K, then of V, 128-byte swizzle) -> f16 K and
+// V tiles in the grouped layout, one hardware conversion per two codes (exact: 3 mantissa bits,
+// exponents within f16's normal range); the power-of-two scales are applied by the consumers.  The
+// four warps of a warpgroup share a tile: warp w decodes key rows 16 w .. 16 w + 15 (8-row groups
+// 2 w, 2 w + 1) of K and of V.  Lane l takes 16-byte chunk c = l & 7 (dims 16c..16c+15) of rows
+// 16 w + 4 i + (l >> 3), i = 0..3: rows 8k + r0 (even i) and 8k + 4 + r0 (odd i) take fixed
+// swizzles, so every address is one of four per-lane bases plus a constant.  All eight loads of a
+// lane go out before any conversion or store, so that their latencies overlap (K then V quarters one
+// after the other measured 1% slower on the hybrid tree).
+__device__ __forceinline__ void decode_e4m3_quarter_kv(uint32_t src, uint32_t dk, uint32_t dv, int lane, int w) {
   const uint32_t c = lane & 7, r0 = lane >> 3;
   const uint32_t s_even = src + r0 * 128 + ((c ^ r0) << 4);
   const uint32_t s_odd = src + (r0 + 4) * 128 + ((c ^ (r0 + 4)) << 4);
   const uint32_t dh = (c >> 2) * kGroupHalfBytes;
-  const uint32_t d_even0 = dst + dh + r0 * 128 + ((((2 * c) & 7) ^ r0) << 4);
-  const uint32_t d_even1 = dst + dh + r0 * 128 + ((((2 * c + 1) & 7) ^ r0) << 4);
-  const uint32_t d_odd0 = dst + dh + (r0 + 4) * 128 + ((((2 * c) & 7) ^ (r0 + 4)) << 4);
-  const uint32_t d_odd1 = dst + dh + (r0 + 4) * 128 + ((((2 * c + 1) & 7) ^ (r0 + 4)) << 4);
+  const uint32_t e0 = dh + r0 * 128 + ((((2 * c) & 7) ^ r0) << 4);
+  const uint32_t e1 = dh + r0 * 128 + ((((2 * c + 1) & 7) ^ r0) << 4);
+  const uint32_t o0 = dh + (r0 + 4) * 128 + ((((2 * c) & 7) ^ (r0 + 4)) << 4);
+  const uint32_t o1 = dh + (r0 + 4) * 128 + ((((2 * c + 1) & 7) ^ (r0 + 4)) << 4);
   const uint32_t k0 = 2 * static_cast<uint32_t>(w);
-  uint4 v[4];
+  uint4 v[8];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) v[i] = lds128((i & 1 ? s_odd : s_even) + (k0 + (i >> 1)) * 1024);
+  for (int i = 0; i < 8; ++i)
+    v[i] = lds128((i & 1 ? s_odd : s_even) + (k0 + ((i >> 1) & 1)) * 1024 + (i >> 2) * (kLandBytes / 2));
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const uint32_t k = k0 + (i >> 1);
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t k = k0 + ((i >> 1) & 1);
+    const uint32_t dst = i < 4 ? dk : dv;
     const uint32_t ws[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
     uint32_t o[8];
 #pragma unroll
@@ -384,8 +387,8 @@ __device__ __forceinline__ void decode_e4m3_quarter(uint32_t src, uint32_t dst, 
           "cvt.rn.f16x2.e4m3x2 %0, lo;\n\tcvt.rn.f16x2.e4m3x2 %1, hi;\n\t}"
           : "=r"(o[2 * q]), "=r"(o[2 * q + 1])
           : "r"(ws[q]));
-    sts128((i & 1 ? d_odd0 : d_even0) + k * kGroupBytes, make_uint4(o[0], o[1], o[2], o[3]));
-    sts128((i & 1 ? d_odd1 : d_even1) + k * kGroupBytes, make_uint4(o[4], o[5], o[6], o[7]));
+    sts128(dst + (i & 1 ? o0 : e0) + k * kGroupBytes, make_uint4(o[0], o[1], o[2], o[3]));
+    sts128(dst + (i & 1 ? o1 : e1) + k * kGroupBytes, make_uint4(o[4], o[5], o[6], o[7]));
   }
 }
 
@@ -470,9 +473,8 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
              mbar_wait(smem_addr(&sm.vempty[y % NV]), ((y / NV) & 1) ^ 1u, p.err, p.wait_ns);
       if (good) {
         const uint32_t src = smem_addr(sm.land + static_cast<size_t>(ls) * kLandBytes);
-        decode_e4m3_quarter(src, smem_addr(sm.kring + static_cast<size_t>(y % NK) * kKVBytes), lane, quarter);
-        decode_e4m3_quarter(src + kLandBytes / 2, smem_addr(sm.vring + static_cast<size_t>(y % NV) * kKVBytes),
-                            lane, quarter);
+        decode_e4m3_quarter_kv(src, smem_addr(sm.kring + static_cast<size_t>(y % NK) * kKVBytes),
+                               smem_addr(sm.vring + static_cast<size_t>(y % NV) * kKVBytes), lane, quarter);
         fence_proxy_async_smem();  // the MMAs read the tiles through the async proxy
       }
     }
