@@ -32,9 +32,11 @@
 // 16-token pages takes 4 boxes per tensor instead of 8.  Ring depths (5 K,
 // 6 V) were measured on GB300: the bytes in flight per SM that the rings
 // allow bound how fast one CTA streams.
-// fp8 target cache (dense and spread rows, when forced): the producer warps
-// land the e4m3 codes in slots of their own and decode them into f16 tiles;
-// q and the draft tiles are converted to f16 and the MMAs multiply in f16.
+// fp8 target cache (dense and spread rows; the default for 17..128 rows): the
+// producer warps land the e4m3 codes of each tile in a landing slot, and the
+// softmax warpgroup between tiles decodes them into the f16 K and V ring tiles
+// (three tiles ahead of the tile it takes next); q and the draft tiles are
+// converted to f16 by the producers and the MMAs multiply in f16.
 #include <cuda_fp16.h>
 
 #include "kvshot_attn_common.cuh"
@@ -60,12 +62,12 @@ constexpr int kBarSoftmax = 1;             // named barrier among the softmax wa
 constexpr uint32_t kTmemCols = 512;        // S0..S3 [0,256), O0 [256,384), O1 [384,512)
 constexpr uint32_t kTmemO = kNS * kTileKeys;
 constexpr int kMiscInts = 20;
-// fp8 (e4m3) target cache: rings of bf16 tiles decoded by the producer warps, which land the codes in two
-// slots of their own (8 KB of K codes and 8 KB of V codes each).
+// fp8 (e4m3) target cache: rings of f16 tiles, decoded by the softmax warpgroups from landing slots
+// that the producer warps fill (8 KB of K codes and 8 KB of V codes each).
 constexpr int kF8NK = 3;
 constexpr int kF8NV = 4;
 constexpr int kLandBytes = 2 * kTileKeys * 128;  // one landing slot: a tile's K codes then its V codes
-constexpr int kLandSlots = 4;                    // tile t lands in slot t % 4, freed when it is decoded
+constexpr int kLandSlots = 4;                    // tile t lands in slot t % kLandSlots, freed when it is decoded
 constexpr int kDecodeAhead = 3;                  // the softmax warpgroup done with tile t decodes tile t + 3
 constexpr int kBarDecode0 = 2;                   // named barriers 2, 3: the 128 threads of warpgroup 0, 1
 static_assert(kLandSlots % 2 == 0, "a landing slot must stay with one producer warp (t and t - kLandSlots)");
