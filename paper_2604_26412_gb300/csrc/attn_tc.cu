@@ -61,7 +61,7 @@ constexpr int kSoftmaxThreads = 256;       // two warpgroups
 constexpr int kBarSoftmax = 1;             // named barrier among the softmax warps
 constexpr uint32_t kTmemCols = 512;        // S0..S3 [0,256), O0 [256,384), O1 [384,512)
 constexpr uint32_t kTmemO = kNS * kTileKeys;
-constexpr int kMiscInts = 20;
+constexpr int kMiscInts = 22;
 // fp8 (e4m3) target cache: rings of f16 tiles, decoded by the softmax warpgroups from landing slots
 // that the producer warps fill (8 KB of K codes and 8 KB of V codes each).
 constexpr int kF8NK = 3;
@@ -203,7 +203,8 @@ struct Smem {
                        // [8..9] / [10..11] K / V tiles issued per producer warp, [12..13] fp8: tiles of
                        // parity 0 / 1 whose landing was issued, [14..15] fp8: of those, tiles whose landing a
                        // decoder waited, [1] fp8: q blocks converted, [16..17] / [18..19] fp8: draft tiles
-                       // landed / converted per producer warp
+                       // landed / converted per producer warp, [20..21] fp8: tiles of parity 0 / 1 decoded (or
+                       // passed through), a count that only grows
   int* len;
   int* base;
   int* lkind;          // fp8 cache: [kLandSlots] 1 when the slot's tile is a draft tile (nothing to decode)
@@ -491,6 +492,7 @@ __device__ __forceinline__ void run_softmax(const AttnParams& p, const Smem& sm,
         mbar_arrive(smem_addr(&sm.lfree[ls]));
         sm.misc[14 + (y & 1)] = (y >> 1) + 1;
       }
+      reinterpret_cast<volatile int*>(sm.misc)[20 + (y & 1)] = (y >> 1) + 1;  // tile y decoded
     }
   };
   // Outputs and the workspace are written only once the preceding kernel has ended
@@ -1077,7 +1079,24 @@ __device__ __forceinline__ void run_producer_f8(const AttnParams& p, const Tenso
     if (draft) {
       const int kslot = t % NK, vslot = t % NV;
       int good = 1;
-      if (lane < 2) {
+      // This warp waits for the ring slots only at its draft tiles, so by itself it cannot know that the
+      // slots' earlier releases have happened (a wait by parity could then pass two phases early).  Tile
+      // t - 1 being decoded means its decoder had seen S of tile t - 4: QK^T of tile t - 4 and P.V of
+      // tile t - 8 had completed, which makes the waits below unambiguous.  A growing count, not a
+      // barrier phase, so the poll cannot be ambiguous itself.
+      if (t >= 1) {
+        const int need = ((t - 1) >> 1) + 1;
+        volatile int* dec = &sm.misc[20 + ((t - 1) & 1)];
+        const uint64_t t0 = global_timer_ns();
+        while (good && *dec < need) {
+          if (*pipe.abort) good = 0;
+          else if (global_timer_ns() - t0 > p.wait_ns) {
+            set_error(p.err, KVSHOT_ERR_TIMEOUT);
+            good = 0;
+          }
+        }
+      }
+      if (lane < 2 && good) {
         const uint32_t bar = lane == 0 ? smem_addr(&sm.kempty[kslot]) : smem_addr(&sm.vempty[vslot]);
         const uint32_t par = ((t / (lane == 0 ? NK : NV)) & 1) ^ 1u;
         good = mbar_wait(bar, par, p.err, p.wait_ns) && !*pipe.abort;
